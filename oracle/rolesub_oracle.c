@@ -1,0 +1,343 @@
+/*
+ * rolesub_oracle.c -- fp64 CPU oracle for RoleSub's value routing and for
+ * attention over the routed values.
+ *
+ * TEST INFRASTRUCTURE ONLY. It is called by the test-suite, by the smoke
+ * check and by the CPU-baseline leg of the benchmark. The CUDA library never
+ * links, loads or calls it, and the two share no code, header, table or
+ * helper. Everything here is plain double-precision loops, written to be
+ * checked against the paper by eye:
+ *
+ *   Sec. 3.2  z = R^T v; z split into S equal groups of d_s = d_v / S;
+ *             a 0/1 mask m with sum_s m_s = K_i keeps K_i groups;
+ *             the routed value is v~ = R M R^T v.
+ *   Sec. 3.3  Eq. (latentrole): a = softmax(f_role(h)), f_role linear here.
+ *   Sec. 3.4  Eq. (routingscore): the group score combines the token state h,
+ *             the role vector a and the pooled language context; this file
+ *             uses the concatenation form gamma = W2 ReLU(W1 [h; a_r a; a_l c]
+ *             + b1) + b2 with c the mean of the episode's retained language
+ *             hidden states; the K_i largest scores are kept (ties: lower
+ *             group index first).
+ *   Attention (Sec. 3, keys and queries unchanged; values routed):
+ *             s_j = q . k_j * scale, p = softmax_j(s) over every cache token
+ *             of the episode (non-causal), o = sum_j p_j v~_j, evaluated as
+ *             o = R_h sum_j p_j M_j z_j (R_h and the sum commute).
+ *
+ * The value space is per head: R = blockdiag(R_1 .. R_H) with group s of a
+ * head holding head dims [s*d_s, (s+1)*d_s); one mask per token is shared by
+ * all heads. Packed storage follows the cache layout documented with the
+ * library (segments episode-major, kinds vis, lang, prop, act; a segment of n
+ * tokens keeping k groups holds [H][n][k][d_s] values and [n][k] indices);
+ * the offsets are recomputed here independently by oracle_layout().
+ */
+#include <math.h>
+#include <stddef.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define OR_KINDS 4
+
+/* Segment offsets of one layer. Segment e*4+kind. Sizes: rows n, packed
+ * H*n*k*d_s values, indices n*k bytes. Returns 0, or -1 on bad arguments. */
+int oracle_layout(int E, int H, int dh, int G, const int *n_tok, const int *k,
+                  long long *row_off, long long *packed_off, long long *idx_off,
+                  long long *totals)
+{
+    if (E < 0 || H <= 0 || dh <= 0 || G <= 0 || dh % G != 0) return -1;
+    long long ds = dh / G;
+    long long r = 0, p = 0, x = 0;
+    for (int e = 0; e < E; ++e) {
+        for (int m = 0; m < OR_KINDS; ++m) {
+            int s = e * OR_KINDS + m;
+            int n = n_tok[s], kk = k[s];
+            if (n < 0 || kk < 0 || kk > G) return -1;
+            row_off[s] = r;
+            packed_off[s] = p;
+            idx_off[s] = x;
+            r += n;
+            p += (long long)H * n * kk * ds;
+            x += (long long)n * kk;
+        }
+    }
+    totals[0] = r;
+    totals[1] = p;
+    totals[2] = x;
+    return 0;
+}
+
+/* Pool of Sec. 3.4: mean of the retained language hidden states; an empty
+ * language set gives c = 0. */
+void oracle_lang_pool(int d, int n_lang, const double *h_lang, double *c)
+{
+    for (int t = 0; t < d; ++t) c[t] = 0.0;
+    if (n_lang <= 0) return;
+    for (int j = 0; j < n_lang; ++j)
+        for (int t = 0; t < d; ++t) c[t] += h_lang[(size_t)j * d + t];
+    for (int t = 0; t < d; ++t) c[t] /= (double)n_lang;
+}
+
+/* Eq. (latentrole): a = softmax(W_re h + b_re), W_re is [C][d]. */
+void oracle_role(int d, int C, const double *W_re, const double *b_re,
+                 const double *h, double *a)
+{
+    double mx = -INFINITY;
+    for (int r = 0; r < C; ++r) {
+        double s = b_re[r];
+        for (int t = 0; t < d; ++t) s += W_re[(size_t)r * d + t] * h[t];
+        a[r] = s;
+        if (s > mx) mx = s;
+    }
+    double z = 0.0;
+    for (int r = 0; r < C; ++r) {
+        a[r] = exp(a[r] - mx);
+        z += a[r];
+    }
+    for (int r = 0; r < C; ++r) a[r] /= z;
+}
+
+/* Eq. (routingscore), concatenation reading:
+ *   x = [h (d) ; alpha_role * a (C) ; alpha_lang * c (d)]
+ *   u = max(0, W1 x + b1)        W1 is [F][2d + C]
+ *   gamma = W2 u + b2            W2 is [G][F]                              */
+void oracle_router_score(int d, int C, int F, int G,
+                         const double *W1, const double *b1,
+                         const double *W2, const double *b2,
+                         const double *h, const double *a, const double *c,
+                         double alpha_role, double alpha_lang, double *gamma)
+{
+    int in = 2 * d + C;
+    double *x = (double *)malloc(sizeof(double) * (size_t)in);
+    double *u = (double *)malloc(sizeof(double) * (size_t)F);
+    for (int t = 0; t < d; ++t) x[t] = h[t];
+    for (int r = 0; r < C; ++r) x[d + r] = alpha_role * a[r];
+    for (int t = 0; t < d; ++t) x[d + C + t] = alpha_lang * c[t];
+    for (int f = 0; f < F; ++f) {
+        double s = b1[f];
+        for (int t = 0; t < in; ++t) s += W1[(size_t)f * in + t] * x[t];
+        u[f] = s > 0.0 ? s : 0.0;
+    }
+    for (int g = 0; g < G; ++g) {
+        double s = b2[g];
+        for (int f = 0; f < F; ++f) s += W2[(size_t)g * F + f] * u[f];
+        gamma[g] = s;
+    }
+    free(x);
+    free(u);
+}
+
+/* Top-K_i of Sec. 3.4. Groups are ranked by (gamma descending, index
+ * ascending); the first k are kept and written in ascending index order.
+ * margin = gamma_(k) - gamma_(k+1) (r-th largest); k = 0 or k = G gives
+ * +infinity (nothing to decide). */
+void oracle_topk(int G, int k, const double *gamma, unsigned char *idx,
+                 double *margin)
+{
+    int order[64];
+    for (int g = 0; g < G; ++g) order[g] = g;
+    /* selection sort by the ranking rule */
+    for (int i = 0; i < G; ++i) {
+        int best = i;
+        for (int j = i + 1; j < G; ++j) {
+            int a = order[j], b = order[best];
+            if (gamma[a] > gamma[b] || (gamma[a] == gamma[b] && a < b)) best = j;
+        }
+        int t = order[i];
+        order[i] = order[best];
+        order[best] = t;
+    }
+    int keep[64];
+    for (int g = 0; g < G; ++g) keep[g] = 0;
+    for (int i = 0; i < k; ++i) keep[order[i]] = 1;
+    int w = 0;
+    for (int g = 0; g < G; ++g)
+        if (keep[g]) idx[w++] = (unsigned char)g;
+    if (margin) {
+        if (k <= 0 || k >= G) *margin = INFINITY;
+        else *margin = gamma[order[k - 1]] - gamma[order[k]];
+    }
+}
+
+/* Sec. 3.2: z = R^T v for one head, R is [dh][dh] row-major (R[m][n]). */
+void oracle_rotate(int dh, const double *R, const double *v, double *z)
+{
+    for (int n = 0; n < dh; ++n) {
+        double s = 0.0;
+        for (int m = 0; m < dh; ++m) s += R[(size_t)m * dh + n] * v[m];
+        z[n] = s;
+    }
+}
+
+/*
+ * Compress one episode of one layer.
+ *   n_tok[4], k[4]          tokens and kept groups of the episode's segments
+ *   packed_off[4], idx_off[4]  where those segments live in the layer
+ *   h_ep, v_ep              [n_cache][d] rows of the episode (kind order)
+ *   R                       [H][dh][dh] of the layer
+ *   W_re [C][d], b_re [C], W1 [F][2d+C], b1 [F], W2 [G][F], b2 [G]
+ *   idx_force               NULL, or the layer's index array to use instead
+ *                           of the router (tests of arbitrary masks)
+ * Outputs (layer arrays are indexed with the offsets above):
+ *   packed_layer, idx_layer; optionally gamma_ep [n_cache][G] (NaN where the
+ *   router does not run), margin_ep [n_cache], z_ep [n_cache][d].
+ * Returns 0, or -1 on bad arguments / forced indices out of range.
+ */
+int oracle_compress_episode(int H, int dh, int G, int C, int F,
+                            const int *n_tok, const int *k,
+                            const long long *packed_off, const long long *idx_off,
+                            const double *h_ep, const double *v_ep, const double *R,
+                            const double *W_re, const double *b_re,
+                            const double *W1, const double *b1,
+                            const double *W2, const double *b2,
+                            double alpha_role, double alpha_lang,
+                            const unsigned char *idx_force,
+                            double *packed_layer, unsigned char *idx_layer,
+                            double *gamma_ep, double *margin_ep, double *z_ep)
+{
+    if (H <= 0 || dh <= 0 || G <= 0 || G > 64 || dh % G != 0) return -1;
+    int d = H * dh, ds = dh / G;
+    int row0[OR_KINDS];
+    int nc = 0;
+    for (int m = 0; m < OR_KINDS; ++m) {
+        if (n_tok[m] < 0 || k[m] < 0 || k[m] > G) return -1;
+        row0[m] = nc;
+        nc += n_tok[m];
+    }
+    /* pooled language context of this episode and layer */
+    double *c = (double *)malloc(sizeof(double) * (size_t)d);
+    oracle_lang_pool(d, n_tok[1], h_ep + (size_t)row0[1] * d, c);
+
+    double *a = (double *)malloc(sizeof(double) * (size_t)(C > 0 ? C : 1));
+    double *gam = (double *)malloc(sizeof(double) * (size_t)G);
+    double *z = (double *)malloc(sizeof(double) * (size_t)dh);
+    int rc = 0;
+    for (int m = 0; m < OR_KINDS && rc == 0; ++m) {
+        int n = n_tok[m], kk = k[m];
+        for (int i = 0; i < n; ++i) {
+            int r = row0[m] + i;
+            const double *h = h_ep + (size_t)r * d;
+            const double *v = v_ep + (size_t)r * d;
+            unsigned char *ix = idx_layer + idx_off[m] + (long long)i * kk;
+            double mg = INFINITY;
+            if (gamma_ep)
+                for (int g = 0; g < G; ++g) gamma_ep[(size_t)r * G + g] = NAN;
+            if (idx_force) {
+                const unsigned char *fx = idx_force + idx_off[m] + (long long)i * kk;
+                for (int j = 0; j < kk; ++j) {
+                    if (fx[j] >= G || (j > 0 && fx[j] <= fx[j - 1])) { rc = -1; break; }
+                    ix[j] = fx[j];
+                }
+                if (rc) break;
+            } else if (kk == G) {
+                for (int j = 0; j < G; ++j) ix[j] = (unsigned char)j;
+            } else if (kk > 0) {
+                oracle_role(d, C, W_re, b_re, h, a);
+                oracle_router_score(d, C, F, G, W1, b1, W2, b2, h, a, c,
+                                    alpha_role, alpha_lang, gam);
+                oracle_topk(G, kk, gam, ix, &mg);
+                if (gamma_ep)
+                    for (int g = 0; g < G; ++g) gamma_ep[(size_t)r * G + g] = gam[g];
+            }
+            if (margin_ep) margin_ep[r] = mg;
+            for (int hh = 0; hh < H; ++hh) {
+                oracle_rotate(dh, R + (size_t)hh * dh * dh, v + (size_t)hh * dh, z);
+                if (z_ep)
+                    for (int t = 0; t < dh; ++t) z_ep[(size_t)r * d + (size_t)hh * dh + t] = z[t];
+                /* packed[seg][h][i][j][:] = z[idx_j * ds : +ds] */
+                double *dst = packed_layer + packed_off[m]
+                            + (((long long)hh * n + i) * kk) * ds;
+                for (int j = 0; j < kk; ++j)
+                    for (int t = 0; t < ds; ++t) dst[(long long)j * ds + t] = z[ix[j] * ds + t];
+            }
+        }
+    }
+    free(c);
+    free(a);
+    free(gam);
+    free(z);
+    return rc;
+}
+
+/*
+ * Attention of one episode's query tokens over its routed cache, heads
+ * [head_begin, head_end) of one layer.
+ *   q_ep [n_q][d], K_ep [n_cache][d] (kind order), packed_layer/idx_layer with
+ *   the segment offsets, R [H][dh][dh], scale (<= 0 means 1/sqrt(dh)).
+ *   o_ep [n_q][d]: only the selected heads are written.
+ * Returns 0, or -1 on bad arguments or stored indices out of range.
+ */
+int oracle_attend_episode(int H, int dh, int G, const int *n_tok, const int *k,
+                          const long long *packed_off, const long long *idx_off,
+                          int n_q, const double *q_ep, const double *K_ep,
+                          const double *packed_layer, const unsigned char *idx_layer,
+                          const double *R, double scale,
+                          int head_begin, int head_end, double *o_ep)
+{
+    if (H <= 0 || dh <= 0 || G <= 0 || G > 64 || dh % G != 0) return -1;
+    int d = H * dh, ds = dh / G;
+    if (scale <= 0.0) scale = 1.0 / sqrt((double)dh);
+    int nc = 0;
+    for (int m = 0; m < OR_KINDS; ++m) {
+        if (n_tok[m] < 0 || k[m] < 0 || k[m] > G) return -1;
+        nc += n_tok[m];
+    }
+    /* the routed value of every cache token in rotated space, zeros where a
+     * group was not kept: ztil[j][h][:] = M_j z_{j,h} */
+    for (int m = 0; m < OR_KINDS; ++m) {
+        int n = n_tok[m], kk = k[m];
+        const unsigned char *ix = idx_layer + idx_off[m];
+        for (long long t = 0; t < (long long)n * kk; ++t)
+            if (ix[t] >= G) return -1;
+    }
+    double *s = (double *)malloc(sizeof(double) * (size_t)(nc > 0 ? nc : 1));
+    double *y = (double *)malloc(sizeof(double) * (size_t)dh);
+    double *ztil = (double *)malloc(sizeof(double) * (size_t)dh);
+    for (int hh = head_begin; hh < head_end; ++hh) {
+        const double *Rh = R + (size_t)hh * dh * dh;
+        for (int qi = 0; qi < n_q; ++qi) {
+            const double *qv = q_ep + (size_t)qi * d + (size_t)hh * dh;
+            double *o = o_ep + (size_t)qi * d + (size_t)hh * dh;
+            for (int t = 0; t < dh; ++t) y[t] = 0.0;
+            if (nc > 0) {
+                double mx = -INFINITY;
+                for (int j = 0; j < nc; ++j) {
+                    const double *kv = K_ep + (size_t)j * d + (size_t)hh * dh;
+                    double acc = 0.0;
+                    for (int t = 0; t < dh; ++t) acc += qv[t] * kv[t];
+                    s[j] = acc * scale;
+                    if (s[j] > mx) mx = s[j];
+                }
+                double zsum = 0.0;
+                for (int j = 0; j < nc; ++j) {
+                    s[j] = exp(s[j] - mx);
+                    zsum += s[j];
+                }
+                int j = 0;
+                for (int m = 0; m < OR_KINDS; ++m) {
+                    int n = n_tok[m], kk = k[m];
+                    for (int i = 0; i < n; ++i, ++j) {
+                        double p = s[j] / zsum;
+                        for (int t = 0; t < dh; ++t) ztil[t] = 0.0;
+                        const unsigned char *ix = idx_layer + idx_off[m] + (long long)i * kk;
+                        const double *src = packed_layer + packed_off[m]
+                                          + (((long long)hh * n + i) * kk) * ds;
+                        for (int jj = 0; jj < kk; ++jj)
+                            for (int t = 0; t < ds; ++t)
+                                ztil[ix[jj] * ds + t] = src[(long long)jj * ds + t];
+                        for (int t = 0; t < dh; ++t) y[t] += p * ztil[t];
+                    }
+                }
+            }
+            /* o = R_h y */
+            for (int m = 0; m < dh; ++m) {
+                double acc = 0.0;
+                for (int t = 0; t < dh; ++t) acc += Rh[(size_t)m * dh + t] * y[t];
+                o[m] = acc;
+            }
+        }
+    }
+    free(s);
+    free(y);
+    free(ztil);
+    return 0;
+}

@@ -1,0 +1,481 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Nothing here compares the oracle with itself: each check is a closed form, a
+special case that reduces to a textbook or library routine (numpy / scipy),
+brute-force enumeration on tiny inputs, an invariant stated in the paper
+(Sec. 3.2 losslessness, mask sums) or a value the paper prints (Tables 1, 3).
+"""
+import itertools
+import math
+import os
+
+import numpy as np
+import pytest
+import scipy.special
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden", "kv_fractions.txt")
+
+
+def haar(rng, n):
+    q, r = np.linalg.qr(rng.standard_normal((n, n)))
+    return q * np.sign(np.diag(r))[None, :]
+
+
+def rnd_problem(rng, H=2, dh=16, G=4, C=3, F=8, n_tok=((5, 3, 0, 0),), k=((4, 4, 4, 4),), n_q=(4,),
+                R=None):
+    E = len(n_tok)
+    d = H * dh
+    rows = int(np.sum(n_tok))
+    qrows = int(np.sum(n_q))
+    p = dict(H=H, dh=dh, G=G, C=C, F=F, n_tok=np.array(n_tok), k=np.array(k), n_q=np.array(n_q))
+    p["h"] = rng.standard_normal((rows, d))
+    p["v"] = rng.standard_normal((rows, d))
+    p["K"] = rng.standard_normal((rows, d))
+    p["q"] = rng.standard_normal((qrows, d))
+    p["R"] = np.stack([haar(rng, dh) for _ in range(H)]) if R is None else R
+    p["W_re"] = 0.3 * rng.standard_normal((C, d))
+    p["b_re"] = 0.3 * rng.standard_normal(C)
+    p["W1"] = 0.3 * rng.standard_normal((F, 2 * d + C))
+    p["b1"] = 0.3 * rng.standard_normal(F)
+    p["W2"] = 0.3 * rng.standard_normal((G, F))
+    p["b2"] = 0.3 * rng.standard_normal(G)
+    p["E"] = E
+    return p
+
+
+def run(oracle, p, alpha_role=0.1, alpha_lang=0.1, idx_force=None, scale=0.0):
+    spec = oracle.Spec(p["H"], p["dh"], p["G"], p["C"], p["F"], p["n_tok"], p["k"], p["n_q"])
+    c = oracle.compress_layer(spec, p["h"], p["v"], p["R"], p["W_re"], p["b_re"], p["W1"], p["b1"],
+                              p["W2"], p["b2"], alpha_role, alpha_lang, idx_force=idx_force)
+    o = oracle.attend_layer(spec, p["q"], p["K"], c["packed"], c["idx"], p["R"], scale=scale)
+    return spec, c, o
+
+
+def dense_attention(p, vtil_fn=None, scale=None):
+    """Textbook softmax(q K^T * scale) V per episode and head, numpy only."""
+    H, dh = p["H"], p["dh"]
+    scale = 1.0 / math.sqrt(dh) if scale is None else scale
+    ep_row = np.concatenate([[0], np.cumsum(np.sum(p["n_tok"], 1))])
+    ep_q = np.concatenate([[0], np.cumsum(p["n_q"])])
+    o = np.zeros_like(p["q"])
+    for e in range(p["E"]):
+        r0, r1 = ep_row[e], ep_row[e + 1]
+        q0, q1 = ep_q[e], ep_q[e + 1]
+        for h in range(H):
+            sl = slice(h * dh, (h + 1) * dh)
+            if r1 == r0:
+                continue
+            s = p["q"][q0:q1, sl] @ p["K"][r0:r1, sl].T * scale
+            P = scipy.special.softmax(s, axis=1)
+            V = p["v"][r0:r1, sl] if vtil_fn is None else vtil_fn(e, h, r0, r1)
+            o[q0:q1, sl] = P @ V
+    return o
+
+
+def rel_err(a, b, dh):
+    """max |a-b| per (row, head) relative to the row norm of b."""
+    a = a.reshape(a.shape[0], -1, dh)
+    b = b.reshape(b.shape[0], -1, dh)
+    nrm = np.linalg.norm(b, axis=2, keepdims=True)
+    return float(np.max(np.abs(a - b) / np.maximum(nrm, 1e-300)))
+
+
+# ---------------------------------------------------------------------------
+# Layout and accounting
+# ---------------------------------------------------------------------------
+
+def test_layout_offsets_hand_computed(oracle):
+    n_tok = [[3, 2, 0, 0], [1, 0, 0, 2]]
+    k = [[2, 4, 4, 4], [0, 4, 1, 4]]
+    lay = oracle.layout(n_tok, k, H=2, dh=8, G=4)   # d_s = 2
+    # packed sizes H*n*k*ds: 24, 32, 0, 0 | 0, 0, 0, 32
+    assert list(lay["packed_off"]) == [0, 24, 56, 56, 56, 56, 56, 56]
+    assert lay["packed_elems"] == 88
+    assert list(lay["idx_off"]) == [0, 6, 14, 14, 14, 14, 14, 14]
+    assert lay["idx_bytes"] == 22
+    assert list(lay["row_off"]) == [0, 3, 5, 5, 5, 6, 6, 6]
+    assert lay["rows"] == 8
+
+
+def half_up(x, nd=2):
+    """Round half away from zero, the way the paper's tables print."""
+    f = 10 ** nd
+    return math.floor(x * f + 0.5 + 1e-9) / f
+
+
+def _golden():
+    vis, lang = [], []
+    for line in open(GOLDEN):
+        line = line.split("#")[0].split()
+        if not line:
+            continue
+        if line[0] == "vis":
+            vis.append((int(line[1]), int(line[2]), int(line[3]), float(line[4])))
+        else:
+            lang.append((int(line[1]), float(line[2]), float(line[3])))
+    return vis, lang
+
+
+def test_kv_fractions_reproduce_tables_1_and_3(oracle):
+    H, dh, G = 32, 128, 16
+    d = H * dh
+    vis, lang = _golden()
+    assert len(vis) == 9 and len(lang) == 4
+    for n_keep, n_total, K, pct in vis:
+        lay = oracle.layout([[n_keep, 0, 0, 0]], [[K, G, G, G]], H, dh, G)
+        kv = (n_keep * d + lay["packed_elems"]) / (2.0 * n_total * d)
+        assert half_up(100 * kv) == pytest.approx(pct, abs=1e-9), (n_keep, K)
+    for K, vpct, kvpct in lang:
+        n = 40
+        lay = oracle.layout([[0, n, 0, 0]], [[G, K, G, G]], H, dh, G)
+        v_frac = lay["packed_elems"] / (n * d)
+        kv = (n * d + lay["packed_elems"]) / (2.0 * n * d)
+        assert half_up(100 * v_frac) == pytest.approx(vpct, abs=1e-9)
+        assert half_up(100 * kv) == pytest.approx(kvpct, abs=1e-9)
+
+
+# ---------------------------------------------------------------------------
+# Router pieces
+# ---------------------------------------------------------------------------
+
+def test_lang_pool_mean_closed_form(oracle):
+    n, d = 7, 5
+    h = np.arange(1, n + 1, dtype=float)[:, None] * np.ones((1, d))
+    assert np.array_equal(oracle.lang_pool(h), np.full(d, (n + 1) / 2.0))
+    assert np.array_equal(oracle.lang_pool(np.zeros((0, d))), np.zeros(d))
+
+
+def test_role_is_softmax(oracle):
+    rng = np.random.default_rng(1)
+    C, d = 16, 40
+    W = rng.standard_normal((C, d))
+    b = rng.standard_normal(C)
+    h = rng.standard_normal(d)
+    a = oracle.role(W, b, h)
+    ref = scipy.special.softmax(W @ h + b)
+    assert np.max(np.abs(a - ref)) < 1e-15
+    assert abs(a.sum() - 1.0) < 1e-14
+    # zero network -> uniform role vector, exactly 1/C
+    assert np.array_equal(oracle.role(np.zeros((C, d)), np.zeros(C), h), np.full(C, 1.0 / C))
+    # large logits do not overflow (max-subtracted)
+    a = oracle.role(W * 1e4, b, h)
+    assert np.all(np.isfinite(a)) and abs(a.sum() - 1.0) < 1e-12
+
+
+def test_router_token_block_alone(oracle):
+    rng = np.random.default_rng(2)
+    d, C = 6, 3
+    F = G = d
+    W1 = np.zeros((F, 2 * d + C))
+    W1[:, :d] = np.eye(d)
+    h = rng.standard_normal(d)
+    g = oracle.router_score(W1, np.zeros(F), np.eye(G), np.zeros(G), h, rng.random(C),
+                            rng.standard_normal(d), 0.7, 0.9)
+    assert np.array_equal(g, np.maximum(h, 0.0))
+
+
+def test_router_role_block_alone(oracle):
+    rng = np.random.default_rng(3)
+    d, C = 6, 4
+    F = G = C
+    W1 = np.zeros((F, 2 * d + C))
+    W1[:, d:d + C] = np.eye(C)
+    W_re = rng.standard_normal((C, d))
+    b_re = rng.standard_normal(C)
+    h = rng.standard_normal(d)
+    a = oracle.role(W_re, b_re, h)
+    g = oracle.router_score(W1, np.zeros(F), np.eye(G), np.zeros(G), h, a, rng.standard_normal(d),
+                            0.25, 0.9)
+    assert np.max(np.abs(g - 0.25 * scipy.special.softmax(W_re @ h + b_re))) < 1e-16
+
+
+def test_router_language_block_alone(oracle):
+    rng = np.random.default_rng(4)
+    d, C = 6, 3
+    F = G = d
+    W1 = np.zeros((F, 2 * d + C))
+    W1[:, d + C:] = np.eye(d)
+    h_lang = rng.random((5, d)) + 0.1      # positive: ReLU is the identity
+    c = oracle.lang_pool(h_lang)
+    g = oracle.router_score(W1, np.zeros(F), np.eye(G), np.zeros(G), rng.standard_normal(d),
+                            rng.random(C), c, 0.7, 0.125)
+    assert np.max(np.abs(g - 0.125 * h_lang.mean(0))) < 1e-16
+
+
+def test_router_biases_and_output_layer(oracle):
+    rng = np.random.default_rng(5)
+    d, C, F, G = 4, 2, 5, 3
+    W1 = np.zeros((F, 2 * d + C))
+    b1 = np.array([1.0, -2.0, 0.5, -0.1, 3.0])
+    W2 = rng.standard_normal((G, F))
+    b2 = rng.standard_normal(G)
+    g = oracle.router_score(W1, b1, W2, b2, rng.standard_normal(d), rng.random(C),
+                            rng.standard_normal(d), 0.1, 0.1)
+    u = np.array([1.0, 0.0, 0.5, 0.0, 3.0])           # ReLU(b1) by hand
+    assert np.max(np.abs(g - (W2 @ u + b2))) < 1e-15
+
+
+# ---------------------------------------------------------------------------
+# Top-K_i selection
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("G", [4, 8])
+def test_topk_equals_best_subset_brute_force(oracle, G):
+    rng = np.random.default_rng(G)
+    for _ in range(50):
+        gam = rng.standard_normal(G)
+        for k in range(G + 1):
+            idx, margin = oracle.topk(gam, k)
+            best = max(itertools.combinations(range(G), k), key=lambda s: sum(gam[list(s)]))
+            assert tuple(idx) == tuple(sorted(best))
+            assert list(idx) == sorted(idx) and len(set(idx)) == k
+            srt = np.sort(gam)[::-1]
+            if 0 < k < G:
+                assert margin == srt[k - 1] - srt[k]
+            else:
+                assert margin == math.inf
+
+
+def test_topk_near_ties(oracle):
+    # exact ties: the lower group index wins
+    idx, m = oracle.topk(np.zeros(16), 4)
+    assert list(idx) == [0, 1, 2, 3] and m == 0.0
+    g = np.array([0.5, 0.5 + 5e-5, 0.3, 0.5 + 2e-4, 0.5 + 5e-5, -1.0])
+    idx, m = oracle.topk(g, 1)
+    assert list(idx) == [3] and m == pytest.approx(1.5e-4, abs=1e-15)
+    idx, m = oracle.topk(g, 2)            # tie between 1 and 4 -> 1
+    assert list(idx) == [1, 3] and m == 0.0
+    idx, m = oracle.topk(g, 3)
+    assert list(idx) == [1, 3, 4] and m == pytest.approx(5e-5, abs=1e-15)
+
+
+# ---------------------------------------------------------------------------
+# Rotation (Sec. 3.2)
+# ---------------------------------------------------------------------------
+
+def test_rotate_is_transpose_product(oracle):
+    dh = 8
+    R = np.zeros((dh, dh))
+    for m in range(dh):
+        R[m, (m + 1) % dh] = 1.0          # a cyclic permutation (not symmetric)
+    v = np.arange(dh, dtype=float) + 1
+    # z = R^T v: z_n = v_{n-1}
+    assert np.array_equal(oracle.rotate(R, v), np.roll(v, 1))
+
+
+def test_rotate_preserves_norm(oracle):
+    rng = np.random.default_rng(6)
+    dh, G = 64, 8
+    R = haar(rng, dh)
+    v = rng.standard_normal(dh)
+    z = oracle.rotate(R, v)
+    assert abs(np.linalg.norm(z) - np.linalg.norm(v)) < 1e-12
+    groups = z.reshape(G, -1)
+    assert abs(np.sum(groups ** 2) - v @ v) < 1e-11
+    assert np.max(np.abs(R @ z - v)) < 1e-12        # lossless round trip
+
+
+# ---------------------------------------------------------------------------
+# Whole path invariants
+# ---------------------------------------------------------------------------
+
+def test_all_groups_kept_equals_dense_attention(oracle):
+    rng = np.random.default_rng(7)
+    G = 4
+    p = rnd_problem(rng, n_tok=((5, 3, 0, 0), (2, 4, 1, 0)), k=((G,) * 4, (G,) * 4), n_q=(4, 3))
+    _, c, o = run(oracle, p)
+    assert rel_err(o, dense_attention(p), p["dh"]) <= 1e-10
+
+
+def test_no_groups_kept_gives_zero(oracle):
+    rng = np.random.default_rng(8)
+    p = rnd_problem(rng, n_tok=((5, 3, 0, 0),), k=((0, 0, 0, 0),), n_q=(4,))
+    _, c, o = run(oracle, p)
+    assert c["packed"].size == 0 and np.array_equal(o, np.zeros_like(o))
+
+
+def _vtil(p, idx_of_token):
+    """v~_j = R_h M_j R_h^T v_j materialised per token (numpy)."""
+    dh, G = p["dh"], p["G"]
+    ds = dh // G
+
+    def fn(e, h, r0, r1):
+        out = []
+        Rh = p["R"][h]
+        for r in range(r0, r1):
+            m = np.zeros(dh)
+            for g in idx_of_token[r]:
+                m[g * ds:(g + 1) * ds] = 1.0
+            out.append(Rh @ np.diag(m) @ Rh.T @ p["v"][r, h * dh:(h + 1) * dh])
+        return np.array(out)
+    return fn
+
+
+def test_every_mask_on_tiny_input_equals_dense_over_routed_values(oracle):
+    rng = np.random.default_rng(9)
+    G = 4
+    for k in range(G + 1):
+        p = rnd_problem(rng, H=2, dh=8, G=G, n_tok=((3, 0, 0, 0),), k=((k, G, G, G),), n_q=(2,))
+        subsets = list(itertools.combinations(range(G), k))
+        for masks in itertools.product(subsets, repeat=3):
+            fx = np.array([g for m in masks for g in m], np.uint8)
+            _, c, o = run(oracle, p, idx_force=fx)
+            ref = dense_attention(p, _vtil(p, {r: masks[r] for r in range(3)}))
+            assert np.max(np.abs(o - ref)) <= 1e-12, (k, masks)
+
+
+def test_complement_masks_sum_to_dense(oracle):
+    rng = np.random.default_rng(10)
+    G, n = 8, 6
+    base = rnd_problem(rng, H=2, dh=16, G=G, n_tok=((n, 0, 0, 0),), n_q=(3,))
+    for k in (1, 3, 5):
+        sel = [np.sort(rng.choice(G, k, replace=False)) for _ in range(n)]
+        comp = [np.setdiff1d(np.arange(G), s) for s in sel]
+        p1 = dict(base, k=np.array([[k, G, G, G]]))
+        p2 = dict(base, k=np.array([[G - k, G, G, G]]))
+        _, _, o1 = run(oracle, p1, idx_force=np.concatenate(sel).astype(np.uint8))
+        _, _, o2 = run(oracle, p2, idx_force=np.concatenate(comp).astype(np.uint8))
+        assert rel_err(o1 + o2, dense_attention(base), 16) <= 1e-12
+    # sum over single-group outputs
+    acc = 0
+    for g in range(G):
+        pg = dict(base, k=np.array([[1, G, G, G]]))
+        _, _, og = run(oracle, pg, idx_force=np.full(n, g, np.uint8))
+        acc = acc + og
+    assert rel_err(acc, dense_attention(base), 16) <= 1e-12
+
+
+def test_identity_rotation_zeroes_unkept_value_columns(oracle):
+    # the paper's "plain" control: R = I, no role term
+    rng = np.random.default_rng(11)
+    H, dh, G = 2, 16, 4
+    ds = dh // G
+    p = rnd_problem(rng, H=H, dh=dh, G=G, n_tok=((6, 2, 0, 0),), k=((2, 3, G, G),), n_q=(3,),
+                    R=np.stack([np.eye(dh)] * H))
+    spec, c, o = run(oracle, p, alpha_role=0.0)
+    lay = spec.lay
+    kept = {}
+    for m in range(2):
+        n, k = p["n_tok"][0][m], p["k"][0][m]
+        r0 = lay["row_off"][m]
+        for i in range(n):
+            kept[r0 + i] = c["idx"][lay["idx_off"][m] + i * k: lay["idx_off"][m] + (i + 1) * k]
+
+    def fn(e, h, r0, r1):
+        V = p["v"][r0:r1, h * dh:(h + 1) * dh].copy()
+        for r in range(r0, r1):
+            mask = np.zeros(dh, bool)
+            for g in kept[r]:
+                mask[g * ds:(g + 1) * ds] = True
+            V[r - r0, ~mask] = 0.0
+        return V
+    assert np.max(np.abs(o - dense_attention(p, fn))) <= 1e-12
+
+
+def test_attention_weights_are_softmax_of_scaled_scores(oracle):
+    # R = I, all kept, v_j = e_j: output column j is p_j
+    rng = np.random.default_rng(12)
+    H, dh, G, n = 1, 16, 4, 10
+    p = rnd_problem(rng, H=H, dh=dh, G=G, n_tok=((n, 0, 0, 0),), k=((G,) * 4,), n_q=(5,),
+                    R=np.eye(dh)[None])
+    p["v"] = np.eye(dh)[:n]
+    for scale in (0.0, 0.37):
+        _, _, o = run(oracle, p, scale=scale)
+        s = p["q"] @ p["K"].T * (1 / math.sqrt(dh) if scale == 0.0 else scale)
+        P = scipy.special.softmax(s, axis=1)
+        assert np.max(np.abs(o[:, :n] - P)) < 1e-15
+        assert np.max(np.abs(o[:, n:])) == 0.0
+
+
+def test_token_permutation_invariance(oracle):
+    rng = np.random.default_rng(13)
+    G = 4
+    p = rnd_problem(rng, H=2, dh=16, G=G, n_tok=((7, 3, 0, 0),), k=((2, 1, G, G),), n_q=(4,))
+    _, _, o = run(oracle, p)
+    perm = np.concatenate([rng.permutation(7), 7 + rng.permutation(3)])
+    p2 = dict(p, h=p["h"][perm], v=p["v"][perm], K=p["K"][perm])
+    _, _, o2 = run(oracle, p2)
+    assert np.max(np.abs(o - o2)) < 1e-12
+
+
+def test_group_permutation_equivariance(oracle):
+    rng = np.random.default_rng(14)
+    G, dh, H = 4, 16, 2
+    ds = dh // G
+    p = rnd_problem(rng, H=H, dh=dh, G=G, n_tok=((7, 3, 0, 0),), k=((2, 1, G, G),), n_q=(4,))
+    spec, c, o = run(oracle, p)
+    pi = np.array([2, 0, 3, 1])           # new group s holds old group pi[s]
+    cols = np.concatenate([np.arange(pi[s] * ds, (pi[s] + 1) * ds) for s in range(G)])
+    p2 = dict(p, R=p["R"][:, :, cols], W2=p["W2"][pi], b2=p["b2"][pi])
+    _, c2, o2 = run(oracle, p2)
+    assert np.max(np.abs(o - o2)) < 1e-12
+    # the kept set is relabelled: new group s kept <=> old group pi[s] kept
+    lay = spec.lay
+    for m in range(2):
+        n, k = p["n_tok"][0][m], p["k"][0][m]
+        for i in range(n):
+            a = c["idx"][lay["idx_off"][m] + i * k: lay["idx_off"][m] + (i + 1) * k]
+            b = c2["idx"][lay["idx_off"][m] + i * k: lay["idx_off"][m] + (i + 1) * k]
+            assert sorted(pi[b]) == sorted(a)
+
+
+def test_compress_scores_use_episode_language_mean_only(oracle):
+    rng = np.random.default_rng(15)
+    G = 8
+    p = rnd_problem(rng, H=2, dh=16, G=G, C=3, F=8, n_tok=((4, 3, 0, 0), (2, 5, 0, 0)),
+                    k=((3, 2, G, G), (1, 4, G, G)), n_q=(2, 2))
+    spec, c, _ = run(oracle, p, alpha_role=0.3, alpha_lang=0.6)
+    d = spec.d
+    for e in range(2):
+        r0 = spec.ep_row[e]
+        nv, nl = p["n_tok"][e][0], p["n_tok"][e][1]
+        cl = p["h"][r0 + nv:r0 + nv + nl].mean(0)
+        for r in range(r0, r0 + nv + nl):
+            a = scipy.special.softmax(p["W_re"] @ p["h"][r] + p["b_re"])
+            x = np.concatenate([p["h"][r], 0.3 * a, 0.6 * cl])
+            g = p["W2"] @ np.maximum(p["W1"] @ x + p["b1"], 0) + p["b2"]
+            assert np.max(np.abs(c["gamma"][r] - g)) < 1e-12
+    # language-only score of an episode with no language tokens: c = 0
+    p0 = rnd_problem(rng, H=2, dh=16, G=G, n_tok=((4, 0, 0, 0),), k=((3, G, G, G),), n_q=(1,))
+    _, c0, _ = run(oracle, p0, alpha_role=0.3, alpha_lang=0.6)
+    r = 1
+    a = scipy.special.softmax(p0["W_re"] @ p0["h"][r] + p0["b_re"])
+    x = np.concatenate([p0["h"][r], 0.3 * a, np.zeros(d)])
+    g = p0["W2"] @ np.maximum(p0["W1"] @ x + p0["b1"], 0) + p0["b2"]
+    assert np.max(np.abs(c0["gamma"][r] - g)) < 1e-12
+
+
+def test_packed_values_are_rotated_groups(oracle):
+    rng = np.random.default_rng(16)
+    G, dh, H = 4, 16, 2
+    ds = dh // G
+    p = rnd_problem(rng, H=H, dh=dh, G=G, n_tok=((5, 2, 0, 0),), k=((2, G, G, G),), n_q=(1,))
+    spec, c, _ = run(oracle, p)
+    lay = spec.lay
+    n, k = 5, 2
+    for i in range(n):
+        sel = c["idx"][i * k:(i + 1) * k]
+        for h in range(H):
+            z = p["R"][h].T @ p["v"][i, h * dh:(h + 1) * dh]
+            got = c["packed"][((h * n + i) * k) * ds:((h * n + i) * k + k) * ds]
+            want = np.concatenate([z[g * ds:(g + 1) * ds] for g in sel])
+            assert np.max(np.abs(got - want)) < 1e-12
+    # the language segment keeps every group, indices 0..G-1
+    assert list(c["idx"][lay["idx_off"][1]:lay["idx_off"][1] + G]) == list(range(G))
+
+
+def test_empty_cache_gives_zero_output(oracle):
+    rng = np.random.default_rng(17)
+    p = rnd_problem(rng, n_tok=((0, 0, 0, 0), (3, 1, 0, 0)), k=((2, 2, 4, 4), (2, 2, 4, 4)), n_q=(3, 2))
+    _, _, o = run(oracle, p)
+    assert np.array_equal(o[:3], np.zeros_like(o[:3]))
+    assert np.any(o[3:] != 0)
+
+
+def test_bad_forced_indices_rejected(oracle):
+    rng = np.random.default_rng(18)
+    p = rnd_problem(rng, n_tok=((2, 0, 0, 0),), k=((2, 4, 4, 4),), n_q=(1,))
+    with pytest.raises(ValueError):
+        run(oracle, p, idx_force=np.array([0, 4, 1, 2], np.uint8))   # 4 >= G
+    with pytest.raises(ValueError):
+        run(oracle, p, idx_force=np.array([1, 1, 1, 2], np.uint8))   # not ascending
