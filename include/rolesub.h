@@ -1,0 +1,231 @@
+/*
+ * rolesub.h -- C ABI of the RoleSub hot path on sm_103a (GB300).
+ *
+ * RoleSub (role-conditioned sub-token routing) keeps keys and queries as
+ * they are and compresses the value vectors of retained tokens (Sec. 3):
+ *
+ *   compress (Sec. 3.2-3.4): per retained token i and layer l
+ *     z_i   = R^T v_i                   rotation into the routing space
+ *     a_i   = softmax(W_re h_i + b_re)   latent role, Eq. (latentrole)
+ *     gamma = W2 ReLU(W1 [h_i ; alpha_role a_i ; alpha_lang c] + b1) + b2
+ *             with c the mean hidden state of the episode's retained
+ *             language tokens, Eq. (routingscore) in concatenation form
+ *     keep the K_i groups with the largest gamma (ties: lower index) and
+ *     store only those groups of z_i plus their indices.
+ *   attend: query tokens read full keys and the routed values,
+ *     o = sum_j softmax_j(q.k_j * scale) R M_j R^T v_j
+ *       = R_h sum_j p_j M_j z_j        (accumulated in the rotated space)
+ *
+ * Geometry. d = H * d_h. The orthonormal value rotation is per head,
+ * R = blockdiag(R_1..R_H); group s of head h holds head dims
+ * [s*d_s, (s+1)*d_s), d_s = d_h / S. One group mask per token is shared by
+ * all heads (one score vector gamma in R^S per token, Sec. 3.4).
+ *
+ * Conventions for every entry point:
+ *  - All functions are synchronous on the host for validation and return a
+ *    rolesub_status. Device work is enqueued on the caller's CUDA stream
+ *    (cudaStream_t passed as void*; NULL = legacy default stream) and is
+ *    asynchronous; no entry point synchronises except
+ *    rolesub_get_device_status.
+ *  - The caller owns every buffer. The library allocates no memory and keeps
+ *    no state between calls (one-time per-process lookups aside).
+ *  - Device pointers must be 16-byte aligned; ROLESUB_EINVAL otherwise.
+ *  - Argument errors return ROLESUB_EINVAL (or ROLESUB_EUNSUPPORTED for a
+ *    valid geometry this build does not implement) before anything is
+ *    launched. A failed launch returns ROLESUB_ECUDA.
+ *  - Bad data found on the device (a stored group index >= S, a bounded
+ *    wait that ran out) is recorded in the workspace's status word; the
+ *    kernel skips the offending item and never traps. Read it with
+ *    rolesub_get_device_status.
+ *  - Tensor element type: one dtype per call (shape.dtype) for h, v, R,
+ *    W_re, W1, W2, q, K, packed values and o. Biases are float32.
+ */
+#ifndef ROLESUB_H
+#define ROLESUB_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ROLESUB_VERSION 1
+#define ROLESUB_PLAN_MAGIC 0x42555352u /* "RSUB" */
+#define ROLESUB_NUM_KINDS 4
+#define ROLESUB_MAX_GROUPS 16
+
+typedef enum {
+    ROLESUB_OK = 0,
+    ROLESUB_EINVAL = 1,        /* bad argument or plan; nothing launched      */
+    ROLESUB_EUNSUPPORTED = 2,  /* geometry not implemented; nothing launched  */
+    ROLESUB_ECUDA = 3,         /* CUDA runtime error or failed launch         */
+    ROLESUB_EDEVICE = 4,       /* kernel found bad data (device status word)  */
+    ROLESUB_ETIMEOUT = 5       /* a bounded in-kernel wait gave up            */
+} rolesub_status;
+
+typedef enum { ROLESUB_F32 = 0, ROLESUB_BF16 = 1 } rolesub_dtype;
+
+/* Token types of Sec. 3.1; every episode has one segment of each, in this
+ * order (a segment may be empty). */
+typedef enum { ROLESUB_VIS = 0, ROLESUB_LANG = 1, ROLESUB_PROP = 2, ROLESUB_ACT = 3 } rolesub_kind;
+
+typedef struct {
+    int32_t num_layers;    /* L                                               */
+    int32_t num_heads;     /* H                                               */
+    int32_t head_dim;      /* d_h (d = H * d_h)                               */
+    int32_t num_groups;    /* S, 1..16, divides d_h (Sec. 3.2)                */
+    int32_t role_dim;      /* C, latent role components (Sec. 3.3)            */
+    int32_t router_hidden; /* F, width of the router's hidden layer           */
+    int32_t dtype;         /* rolesub_dtype                                   */
+    int32_t reserved;      /* must be 0                                       */
+} rolesub_shape;
+
+/* One (episode, kind) run of cache rows. Offsets are per layer; layer l's
+ * arrays start at l * {rows,packed_elems,idx_bytes}_per_layer. */
+typedef struct {
+    int32_t episode;
+    int32_t kind;          /* rolesub_kind                                    */
+    int32_t n_tokens;      /* retained tokens of this type (|I_m^keep|)       */
+    int32_t k;             /* kept groups per token K_m, 0..S                 */
+    int64_t token_row;     /* first row of this segment in h / v / K          */
+    int64_t packed_off;    /* element offset of its [H][n_tokens][k][d_s]     */
+    int64_t idx_off;       /* byte offset of its [n_tokens][k] uint8 indices  */
+} rolesub_segment;
+
+typedef struct {
+    int64_t row_begin;     /* first cache row of the episode                  */
+    int64_t q_row_begin;   /* first query row of the episode                  */
+    int32_t n_cache;       /* cache rows (all kinds)                          */
+    int32_t n_query;       /* query rows                                      */
+    int32_t seg_begin;     /* index of its first segment (= 4 * episode)      */
+    int32_t n_lang;        /* retained language tokens                        */
+    int64_t lang_row_begin;
+} rolesub_episode;
+
+/* A plan is one self-contained byte blob: this header followed by the
+ * arrays it points to (byte offsets from the start of the blob). The same
+ * bytes are used on the host (validation, grid sizes) and, copied verbatim
+ * by the caller into device memory, by the kernels. */
+typedef struct {
+    uint32_t magic;                  /* ROLESUB_PLAN_MAGIC                     */
+    uint32_t version;                /* ROLESUB_VERSION                        */
+    int32_t num_episodes;
+    int32_t num_segments;            /* 4 * num_episodes                       */
+    int64_t rows_per_layer;          /* cache rows of every episode            */
+    int64_t q_rows_per_layer;        /* query rows of every episode            */
+    int64_t packed_elems_per_layer;  /* sum over segments of H*n*k*d_s         */
+    int64_t idx_bytes_per_layer;     /* sum over segments of n*k               */
+    int64_t routed_rows_per_layer;   /* rows of segments with 0 < k < S        */
+    int64_t stored_rows_per_layer;   /* rows of segments with k > 0            */
+    int32_t max_cache_tokens;        /* max n_cache over episodes              */
+    int32_t max_query_tokens;        /* max n_query over episodes              */
+    int32_t num_heads, head_dim, num_groups, reserved;  /* geometry checked at use */
+    int64_t off_segments;            /* rolesub_segment[num_segments]          */
+    int64_t off_episodes;            /* rolesub_episode[num_episodes]          */
+    int64_t off_row_seg;             /* int32[rows_per_layer]: segment of row  */
+    int64_t off_routed_rows;         /* int32[routed_rows]: ascending row ids  */
+    int64_t off_stored_rows;         /* int32[stored_rows]: ascending row ids  */
+    int64_t total_bytes;             /* size of the whole blob                 */
+} rolesub_plan;
+
+/* Bytes needed for the plan of num_episodes episodes with n_tok[e*4+kind]
+ * tokens. ROLESUB_EINVAL on negative counts. */
+rolesub_status rolesub_plan_size(int32_t num_episodes, const int32_t *n_tok, size_t *bytes);
+
+/*
+ * Cache layout of Sec. 3.2's packed values (the paper fixes only the
+ * accounting: keys full, K_i of S value groups per token; the layout is this
+ * library's): segments ordered episode-major, kind-minor; segment
+ * (n tokens, k groups) holds values [H][n][k][d_s] at packed_off and indices
+ * [n][k] (ascending group ids, uint8) at idx_off. k = S stores every group
+ * with indices 0..S-1; k = 0 stores nothing.
+ *   n_tok[e*4+m], k[e*4+m]: tokens and kept groups of kind m in episode e
+ *   n_query[e]: query tokens of episode e
+ *   plan / plan_bytes: host output buffer (>= rolesub_plan_size), 16-byte
+ *   aligned. Copy plan->total_bytes of it to a 16-byte-aligned device buffer
+ *   to obtain plan_dev for the calls below.
+ * ROLESUB_EINVAL on k outside 0..S, bad geometry or a short buffer.
+ */
+rolesub_status rolesub_layout_plan(const rolesub_shape *shape, int32_t num_episodes,
+                                   const int32_t *n_tok, const int32_t *k,
+                                   const int32_t *n_query, void *plan, size_t plan_bytes);
+
+/* Scratch bytes a compress or attend call needs (the larger of the two).
+ * The workspace also holds the device status word; zero it once (or call
+ * rolesub_reset_device_status) before the first call that uses it. */
+rolesub_status rolesub_workspace_size(const rolesub_shape *shape, const void *plan_host,
+                                      size_t *bytes);
+
+/*
+ * Routing and packing of every routed token of every layer (Sec. 3.2-3.4).
+ * Inputs (device, dtype = shape.dtype unless noted, row-major contiguous):
+ *   h     [L][rows][d]          hidden states of the cache rows
+ *   v     [L][rows][H][d_h]     value vectors
+ *   R     [L][H][d_h][d_h]      per-head orthonormal rotation (R[m][n])
+ *   W_re  [L][C][d], b_re [L][C] float32    role estimator
+ *   W1    [L][F][2d+C], b1 [L][F] float32   router hidden layer; input
+ *                                            columns [h | role | language]
+ *   W2    [L][S][F],  b2 [L][S]  float32    router output layer
+ *   alpha_role, alpha_lang                   Eq. (routingscore) weights
+ * Outputs (device):
+ *   packed_v [L][packed_elems_per_layer]  dtype; rotated kept groups
+ *   idx      [L][idx_bytes_per_layer]     uint8; kept groups, ascending
+ * workspace / ws_bytes: device scratch (>= rolesub_workspace_size).
+ * Segments with k = 0 write nothing; k = S store every group without
+ * running the router.
+ */
+rolesub_status rolesub_compress(const rolesub_shape *shape, const void *plan_host,
+                                const void *plan_dev, const void *h, const void *v,
+                                const void *R, const void *W_re, const float *b_re,
+                                const void *W1, const float *b1, const void *W2,
+                                const float *b2, float alpha_role, float alpha_lang,
+                                void *packed_v, uint8_t *idx, void *workspace,
+                                size_t ws_bytes, void *stream);
+
+/*
+ * Attention of every episode's query tokens over its own routed cache
+ * (all cache tokens of the episode, non-causal), per layer and head:
+ *   s_j = (q . k_j) * scale, p = softmax_j(s), y = sum_j p_j M_j z_j,
+ *   o = R_h y.
+ * Inputs (device, dtype = shape.dtype):
+ *   q  [L][q_rows][H][d_h], element (l, r, h, t) at
+ *      l*q_layer_stride + r*q_row_stride + h*q_head_stride + t
+ *   K  [L][rows][H][d_h], same addressing with the k_* strides (the
+ *      caller's key cache; read in place). Strides are in elements and must
+ *      be multiples of 8 (16 bytes of bf16; 4 suffice for float32).
+ *   packed_v, idx   as written by rolesub_compress
+ *   R  [L][H][d_h][d_h]
+ *   softmax_scale   0 means 1/sqrt(d_h)
+ * Output: o [L][q_rows][H][d_h] contiguous, dtype.
+ * A cache with no tokens gives o = 0. Stored indices >= S are skipped and
+ * reported through the device status word.
+ */
+rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
+                              const void *plan_dev, const void *q, int64_t q_layer_stride,
+                              int64_t q_row_stride, int64_t q_head_stride, const void *K,
+                              int64_t k_layer_stride, int64_t k_row_stride,
+                              int64_t k_head_stride, const void *packed_v, const uint8_t *idx,
+                              const void *R, float softmax_scale, void *o, void *workspace,
+                              size_t ws_bytes, void *stream);
+
+/* Waits for the stream, then reads the workspace's status word:
+ * *code_out = 0 when no kernel reported bad data, else a ROLESUB_E* code.
+ * *detail_out (may be NULL) receives the first reported item. */
+rolesub_status rolesub_get_device_status(const void *workspace, void *stream, int32_t *code_out,
+                                         int32_t *detail_out);
+
+/* Enqueues a clear of the status word on the stream. */
+rolesub_status rolesub_reset_device_status(void *workspace, void *stream);
+
+/* Static description of a status code. */
+const char *rolesub_status_string(rolesub_status s);
+
+/* ROLESUB_VERSION of the library actually loaded. */
+int32_t rolesub_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ROLESUB_H */

@@ -1,0 +1,359 @@
+// api.cu -- the C ABI of include/rolesub.h: plan construction, argument
+// validation (always before any launch) and the launch sequences.
+#include <math.h>
+#include <string.h>
+
+#include <vector>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace {
+
+using rs::PlanView;
+using rs::Workspace;
+
+constexpr size_t kAlign = 256;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+bool aligned16(const void *p) { return ((uintptr_t)p & 15u) == 0; }
+
+int elem_bytes(int dtype) { return dtype == ROLESUB_BF16 ? 2 : 4; }
+
+bool shape_ok(const rolesub_shape *s)
+{
+    if (!s) return false;
+    if (s->num_layers < 1 || s->num_heads < 1 || s->head_dim < 1) return false;
+    if (s->num_groups < 1 || s->num_groups > ROLESUB_MAX_GROUPS) return false;
+    if (s->head_dim % s->num_groups != 0) return false;
+    if (s->role_dim < 1 || s->router_hidden < 1) return false;
+    if (s->dtype != ROLESUB_F32 && s->dtype != ROLESUB_BF16) return false;
+    if (s->reserved != 0) return false;
+    if ((int64_t)s->num_heads * s->head_dim > (1 << 20)) return false;
+    return true;
+}
+
+struct Sizes {
+    size_t header, segs, eps, row_seg, routed, stored, total;
+};
+
+Sizes plan_sizes(int32_t E, int64_t rows)
+{
+    Sizes z;
+    z.header = align_up(sizeof(rolesub_plan), 16);
+    z.segs = align_up(sizeof(rolesub_segment) * (size_t)E * ROLESUB_NUM_KINDS, 16);
+    z.eps = align_up(sizeof(rolesub_episode) * (size_t)E, 16);
+    z.row_seg = align_up(sizeof(int32_t) * (size_t)rows, 16);
+    z.routed = z.row_seg;
+    z.stored = z.row_seg;
+    z.total = z.header + z.segs + z.eps + z.row_seg + z.routed + z.stored;
+    return z;
+}
+
+// Validates a plan blob against a shape and fills the host view.
+rolesub_status view_plan(const rolesub_shape *s, const void *plan_host, const void *plan_dev,
+                         PlanView *pv)
+{
+    if (!plan_host || !aligned16(plan_host)) return ROLESUB_EINVAL;
+    const rolesub_plan *p = (const rolesub_plan *)plan_host;
+    if (p->magic != ROLESUB_PLAN_MAGIC || p->version != ROLESUB_VERSION) return ROLESUB_EINVAL;
+    if (p->num_heads != s->num_heads || p->head_dim != s->head_dim ||
+        p->num_groups != s->num_groups)
+        return ROLESUB_EINVAL;
+    if (p->num_episodes < 0 || p->num_segments != p->num_episodes * ROLESUB_NUM_KINDS)
+        return ROLESUB_EINVAL;
+    if (p->rows_per_layer >= (int64_t)1 << 31) return ROLESUB_EUNSUPPORTED;
+    if (plan_dev && !aligned16(plan_dev)) return ROLESUB_EINVAL;
+    const char *b = (const char *)plan_host;
+    pv->hdr = p;
+    pv->segs = (const rolesub_segment *)(b + p->off_segments);
+    pv->eps = (const rolesub_episode *)(b + p->off_episodes);
+    const char *d = (const char *)plan_dev;
+    pv->dev = d;
+    pv->segs_dev = d ? (const rolesub_segment *)(d + p->off_segments) : nullptr;
+    pv->eps_dev = d ? (const rolesub_episode *)(d + p->off_episodes) : nullptr;
+    pv->row_seg_dev = d ? (const int32_t *)(d + p->off_row_seg) : nullptr;
+    pv->routed_dev = d ? (const int32_t *)(d + p->off_routed_rows) : nullptr;
+    pv->stored_dev = d ? (const int32_t *)(d + p->off_stored_rows) : nullptr;
+    return ROLESUB_OK;
+}
+
+struct WsSizes {
+    size_t status, ctx, bias, logits, total;
+};
+
+WsSizes ws_sizes(const rolesub_shape *s, const rolesub_plan *p)
+{
+    WsSizes w;
+    const size_t L = s->num_layers, E = p->num_episodes;
+    const size_t d = (size_t)s->num_heads * s->head_dim;
+    w.status = rs::kStatusBytes;
+    w.ctx = align_up(sizeof(float) * L * E * d, kAlign);
+    w.bias = align_up(sizeof(float) * L * E * s->router_hidden, kAlign);
+    w.logits = align_up(sizeof(float) * L * (size_t)p->routed_rows_per_layer *
+                            (size_t)(s->router_hidden + s->role_dim),
+                        kAlign);
+    w.total = w.status + w.ctx + w.bias + w.logits;
+    return w;
+}
+
+Workspace carve(const WsSizes &w, void *base)
+{
+    Workspace ws;
+    char *b = (char *)base;
+    ws.status = (int32_t *)b;
+    ws.lang_ctx = (float *)(b + w.status);
+    ws.lang_bias = (float *)(b + w.status + w.ctx);
+    ws.logits = (float *)(b + w.status + w.ctx + w.bias);
+    ws.bytes = w.total;
+    return ws;
+}
+
+rolesub_status from_cuda(cudaError_t e) { return e == cudaSuccess ? ROLESUB_OK : ROLESUB_ECUDA; }
+
+}  // namespace
+
+extern "C" {
+
+int32_t rolesub_version(void) { return ROLESUB_VERSION; }
+
+const char *rolesub_status_string(rolesub_status s)
+{
+    switch (s) {
+    case ROLESUB_OK: return "ok";
+    case ROLESUB_EINVAL: return "invalid argument";
+    case ROLESUB_EUNSUPPORTED: return "unsupported geometry";
+    case ROLESUB_ECUDA: return "CUDA error";
+    case ROLESUB_EDEVICE: return "bad data found on the device";
+    case ROLESUB_ETIMEOUT: return "in-kernel wait timed out";
+    }
+    return "unknown status";
+}
+
+rolesub_status rolesub_plan_size(int32_t num_episodes, const int32_t *n_tok, size_t *bytes)
+{
+    if (num_episodes < 0 || !bytes || (num_episodes > 0 && !n_tok)) return ROLESUB_EINVAL;
+    int64_t rows = 0;
+    for (int64_t i = 0; i < (int64_t)num_episodes * ROLESUB_NUM_KINDS; ++i) {
+        if (n_tok[i] < 0) return ROLESUB_EINVAL;
+        rows += n_tok[i];
+    }
+    *bytes = plan_sizes(num_episodes, rows).total;
+    return ROLESUB_OK;
+}
+
+rolesub_status rolesub_layout_plan(const rolesub_shape *shape, int32_t E, const int32_t *n_tok,
+                                   const int32_t *k, const int32_t *n_query, void *plan,
+                                   size_t plan_bytes)
+{
+    if (!shape_ok(shape) || E < 0 || !plan || !aligned16(plan)) return ROLESUB_EINVAL;
+    if (E > 0 && (!n_tok || !k || !n_query)) return ROLESUB_EINVAL;
+    const int G = shape->num_groups, H = shape->num_heads;
+    const int64_t ds = shape->head_dim / G;
+    int64_t rows = 0, qrows = 0;
+    for (int64_t i = 0; i < (int64_t)E * ROLESUB_NUM_KINDS; ++i) {
+        if (n_tok[i] < 0 || k[i] < 0 || k[i] > G) return ROLESUB_EINVAL;
+        rows += n_tok[i];
+    }
+    for (int e = 0; e < E; ++e) {
+        if (n_query[e] < 0) return ROLESUB_EINVAL;
+        qrows += n_query[e];
+    }
+    const Sizes z = plan_sizes(E, rows);
+    if (plan_bytes < z.total) return ROLESUB_EINVAL;
+    memset(plan, 0, z.total);
+    char *b = (char *)plan;
+    rolesub_plan *p = (rolesub_plan *)b;
+    p->magic = ROLESUB_PLAN_MAGIC;
+    p->version = ROLESUB_VERSION;
+    p->num_episodes = E;
+    p->num_segments = E * ROLESUB_NUM_KINDS;
+    p->num_heads = H;
+    p->head_dim = shape->head_dim;
+    p->num_groups = G;
+    p->off_segments = (int64_t)z.header;
+    p->off_episodes = (int64_t)(z.header + z.segs);
+    p->off_row_seg = (int64_t)(z.header + z.segs + z.eps);
+    p->off_routed_rows = p->off_row_seg + (int64_t)z.row_seg;
+    p->off_stored_rows = p->off_routed_rows + (int64_t)z.routed;
+    p->total_bytes = (int64_t)z.total;
+    rolesub_segment *segs = (rolesub_segment *)(b + p->off_segments);
+    rolesub_episode *eps = (rolesub_episode *)(b + p->off_episodes);
+    int32_t *row_seg = (int32_t *)(b + p->off_row_seg);
+    int32_t *routed = (int32_t *)(b + p->off_routed_rows);
+    int32_t *stored = (int32_t *)(b + p->off_stored_rows);
+    int64_t r = 0, qr = 0, pk = 0, ix = 0, nrouted = 0, nstored = 0;
+    int32_t max_c = 0, max_q = 0;
+    for (int e = 0; e < E; ++e) {
+        rolesub_episode &ep = eps[e];
+        ep.row_begin = r;
+        ep.q_row_begin = qr;
+        ep.n_query = n_query[e];
+        ep.seg_begin = e * ROLESUB_NUM_KINDS;
+        int32_t nc = 0;
+        for (int m = 0; m < ROLESUB_NUM_KINDS; ++m) {
+            const int s = e * ROLESUB_NUM_KINDS + m;
+            rolesub_segment &sg = segs[s];
+            sg.episode = e;
+            sg.kind = m;
+            sg.n_tokens = n_tok[s];
+            sg.k = k[s];
+            sg.token_row = r;
+            sg.packed_off = pk;
+            sg.idx_off = ix;
+            if (m == ROLESUB_LANG) {
+                ep.n_lang = n_tok[s];
+                ep.lang_row_begin = r;
+            }
+            for (int i = 0; i < n_tok[s]; ++i) {
+                row_seg[r + i] = s;
+                if (k[s] > 0) stored[nstored++] = (int32_t)(r + i);
+                if (k[s] > 0 && k[s] < G) routed[nrouted++] = (int32_t)(r + i);
+            }
+            r += n_tok[s];
+            nc += n_tok[s];
+            pk += (int64_t)H * n_tok[s] * k[s] * ds;
+            ix += (int64_t)n_tok[s] * k[s];
+        }
+        ep.n_cache = nc;
+        if (nc > max_c) max_c = nc;
+        if (n_query[e] > max_q) max_q = n_query[e];
+        qr += n_query[e];
+    }
+    p->rows_per_layer = r;
+    p->q_rows_per_layer = qr;
+    p->packed_elems_per_layer = pk;
+    p->idx_bytes_per_layer = ix;
+    p->routed_rows_per_layer = nrouted;
+    p->stored_rows_per_layer = nstored;
+    p->max_cache_tokens = max_c;
+    p->max_query_tokens = max_q;
+    return ROLESUB_OK;
+}
+
+rolesub_status rolesub_workspace_size(const rolesub_shape *shape, const void *plan_host,
+                                      size_t *bytes)
+{
+    if (!shape_ok(shape) || !bytes) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, nullptr, &pv);
+    if (st != ROLESUB_OK) return st;
+    *bytes = ws_sizes(shape, pv.hdr).total;
+    return ROLESUB_OK;
+}
+
+rolesub_status rolesub_compress(const rolesub_shape *shape, const void *plan_host,
+                                const void *plan_dev, const void *h, const void *v,
+                                const void *R, const void *W_re, const float *b_re,
+                                const void *W1, const float *b1, const void *W2,
+                                const float *b2, float alpha_role, float alpha_lang,
+                                void *packed_v, uint8_t *idx, void *workspace, size_t ws_bytes,
+                                void *stream)
+{
+    if (!shape_ok(shape)) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, plan_dev, &pv);
+    if (st != ROLESUB_OK) return st;
+    if (!plan_dev) return ROLESUB_EINVAL;
+    const void *ptrs[] = {h, v, R, W_re, b_re, W1, b1, W2, b2, workspace};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    const rolesub_plan &P = *pv.hdr;
+    if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
+    if (P.idx_bytes_per_layer > 0 && (!idx || !aligned16(idx))) return ROLESUB_EINVAL;
+    if (!isfinite(alpha_role) || !isfinite(alpha_lang)) return ROLESUB_EINVAL;
+    const WsSizes w = ws_sizes(shape, pv.hdr);
+    if (ws_bytes < w.total) return ROLESUB_EINVAL;
+    if (!rs::router_supported(shape) || !rs::rotate_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    rs::CompressArgs a;
+    a.shape = shape;
+    a.plan = pv;
+    a.ws = carve(w, workspace);
+    a.h = h;
+    a.v = v;
+    a.R = R;
+    a.W_re = W_re;
+    a.W1 = W1;
+    a.W2 = W2;
+    a.b_re = b_re;
+    a.b1 = b1;
+    a.b2 = b2;
+    a.alpha_role = alpha_role;
+    a.alpha_lang = alpha_lang;
+    a.packed = packed_v;
+    a.idx = idx;
+    a.stream = (cudaStream_t)stream;
+    cudaError_t e = rs::launch_router(a);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    return from_cuda(rs::launch_rotate_pack(a));
+}
+
+rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
+                              const void *plan_dev, const void *q, int64_t q_ls, int64_t q_rs,
+                              int64_t q_hs, const void *K, int64_t k_ls, int64_t k_rs,
+                              int64_t k_hs, const void *packed_v, const uint8_t *idx,
+                              const void *R, float softmax_scale, void *o, void *workspace,
+                              size_t ws_bytes, void *stream)
+{
+    if (!shape_ok(shape)) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, plan_dev, &pv);
+    if (st != ROLESUB_OK) return st;
+    if (!plan_dev) return ROLESUB_EINVAL;
+    const rolesub_plan &P = *pv.hdr;
+    const void *ptrs[] = {q, K, R, o, workspace};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
+    if (P.idx_bytes_per_layer > 0 && !idx) return ROLESUB_EINVAL;
+    const int64_t sm = 16 / elem_bytes(shape->dtype);
+    const int64_t strides[] = {q_ls, q_rs, q_hs, k_ls, k_rs, k_hs};
+    for (int64_t x : strides)
+        if (x < 0 || x % sm != 0) return ROLESUB_EINVAL;
+    if (!isfinite(softmax_scale) || softmax_scale < 0.f) return ROLESUB_EINVAL;
+    const WsSizes w = ws_sizes(shape, pv.hdr);
+    if (ws_bytes < w.total) return ROLESUB_EINVAL;
+    if (!rs::attend_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    rs::AttendArgs a;
+    a.shape = shape;
+    a.plan = pv;
+    a.ws = carve(w, workspace);
+    a.q = q;
+    a.K = K;
+    a.packed = packed_v;
+    a.R = R;
+    a.idx = idx;
+    a.q_ls = q_ls;
+    a.q_rs = q_rs;
+    a.q_hs = q_hs;
+    a.k_ls = k_ls;
+    a.k_rs = k_rs;
+    a.k_hs = k_hs;
+    a.scale = softmax_scale;
+    a.o = o;
+    a.stream = (cudaStream_t)stream;
+    return from_cuda(rs::launch_attend(a));
+}
+
+rolesub_status rolesub_get_device_status(const void *workspace, void *stream, int32_t *code_out,
+                                         int32_t *detail_out)
+{
+    if (!workspace || !code_out || !aligned16(workspace)) return ROLESUB_EINVAL;
+    int32_t hs[2] = {0, 0};
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaMemcpyAsync(hs, workspace, sizeof(hs), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return ROLESUB_ECUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return ROLESUB_ECUDA;
+    *code_out = hs[0];
+    if (detail_out) *detail_out = hs[1];
+    return ROLESUB_OK;
+}
+
+rolesub_status rolesub_reset_device_status(void *workspace, void *stream)
+{
+    if (!workspace || !aligned16(workspace)) return ROLESUB_EINVAL;
+    return from_cuda(cudaMemsetAsync(workspace, 0, rs::kStatusBytes, (cudaStream_t)stream));
+}
+
+}  // extern "C"

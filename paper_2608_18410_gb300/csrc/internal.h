@@ -1,0 +1,68 @@
+// internal.h -- host-side launchers shared between the C-ABI layer and the
+// kernel translation units. Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "rolesub.h"
+
+namespace rs {
+
+struct PlanView {  // host view of a validated plan + device copy
+    const rolesub_plan *hdr;
+    const rolesub_segment *segs;     // host
+    const rolesub_episode *eps;      // host
+    const char *dev;                 // device copy base
+    const rolesub_segment *segs_dev;
+    const rolesub_episode *eps_dev;
+    const int32_t *row_seg_dev;
+    const int32_t *routed_dev;
+    const int32_t *stored_dev;
+};
+
+struct Workspace {  // carve-up of the caller's workspace
+    int32_t *status;
+    float *lang_ctx;   // [L][E][d]
+    float *lang_bias;  // [L][E][F]
+    float *logits;     // [L][routed][F + C]   (router GEMM output)
+    size_t bytes;
+};
+
+struct CompressArgs {
+    const rolesub_shape *shape;
+    PlanView plan;
+    Workspace ws;
+    const void *h, *v, *R, *W_re, *W1, *W2;
+    const float *b_re, *b1, *b2;
+    float alpha_role, alpha_lang;
+    void *packed;
+    uint8_t *idx;
+    cudaStream_t stream;
+};
+
+struct AttendArgs {
+    const rolesub_shape *shape;
+    PlanView plan;
+    Workspace ws;
+    const void *q, *K, *packed, *R;
+    const uint8_t *idx;
+    int64_t q_ls, q_rs, q_hs, k_ls, k_rs, k_hs;
+    float scale;
+    void *o;
+    cudaStream_t stream;
+};
+
+// Router: language pool + per-episode bias, router GEMM, epilogue/top-k.
+cudaError_t launch_router(const CompressArgs &a);
+// Rotation z = R_h^T v and packing of the kept groups.
+cudaError_t launch_rotate_pack(const CompressArgs &a);
+// Routed attention.
+cudaError_t launch_attend(const AttendArgs &a);
+
+// Limits of this build (checked before any launch).
+bool router_supported(const rolesub_shape *s);
+bool rotate_supported(const rolesub_shape *s);
+bool attend_supported(const rolesub_shape *s);
+
+}  // namespace rs
