@@ -1,0 +1,468 @@
+"""RoleSub hot-path benchmark: compress + attend on synthetic OpenVLA-OFT-7B
+shaped inputs, timed on the GPU with CUDA events.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c1|c2|c3|c4]
+                  [--impl ours|reference]
+
+One step = rolesub_compress + rolesub_attend over every layer and episode of
+the workload (all steps of the path). Prints ONE JSON line on rank 0.
+
+Metric: action-query tokens per second per layer for compress + attend,
+value = (query tokens x layers x ranks) / max-over-ranks time. Per-step
+inputs are larger than L2 for c2-c4; for c1 the L2 is flushed (a 512 MB
+write) between timed steps, outside the timed region.
+
+--impl reference times the fp64 CPU oracle (the plain restatement of the
+paper's method) on the host cores, on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "action-query attend+compress tokens/s per layer; HBM GB/s fraction of peak"
+UNIT = "query tokens/s/layer"
+FLUSH_BYTES = 512 << 20
+
+
+# ---------------------------------------------------------------------------
+# workload and accounting
+# ---------------------------------------------------------------------------
+
+def make_workload(name, rank=0):
+    from paper_2608_18410_gb300 import synth
+    import dataclasses
+    if name == "c2":
+        wl = synth.c2(128, 4)
+    else:
+        wl = synth.WORKLOADS[name]()
+    if rank:
+        wl = dataclasses.replace(wl, seed=wl.seed + 1000 * rank)
+    return wl
+
+
+def attend_bytes(wl):
+    """Algorithmic bytes of one rolesub_attend over the workload.
+
+    Per (layer, episode): q and o (Nq*d each), full keys (Nc*d), packed kept
+    groups (sum_j k_j*H*d_s), their indices (sum_j k_j bytes); R_h once per
+    layer (H*d_h^2). Elements are b bytes (2 for bf16, 4 for fp32).
+    """
+    b = 2 if wl.dtype == "bf16" else 4
+    d, H, ds = wl.d, wl.H, wl.dh // wl.G
+    per_layer = H * wl.dh * wl.dh * b
+    for ep in wl.episodes:
+        ks = sum(n * k for n, k in zip(ep.n_tok(), ep.k(wl.G)))
+        per_layer += 2 * ep.n_query * d * b + ep.n_cache * d * b + ks * H * ds * b + ks
+    return per_layer * wl.L
+
+
+def compress_bytes(wl):
+    """Algorithmic bytes of one rolesub_compress over the workload.
+
+    Per layer: h of routed and language rows, v of stored rows, R, all
+    router weights (W_re, W1, W2, fp32 biases), packed values and indices
+    written.
+    """
+    b = 2 if wl.dtype == "bf16" else 4
+    d, H, ds, G = wl.d, wl.H, wl.dh // wl.G, wl.G
+    per_layer = H * wl.dh * wl.dh * b + (wl.C * d + wl.F * (2 * d + wl.C) + G * wl.F) * b
+    per_layer += 4 * (wl.C + wl.F + G)
+    for ep in wl.episodes:
+        for kind, (n, k) in enumerate(zip(ep.n_tok(), ep.k(G))):
+            routed = 0 < k < G
+            if routed or kind == 1:
+                per_layer += n * d * b
+            if k > 0:
+                per_layer += n * d * b + n * k * H * ds * b + n * k
+    return per_layer * wl.L
+
+
+def attend_flops(wl):
+    d, H, ds = wl.d, wl.H, wl.dh // wl.G
+    f = 0
+    for ep in wl.episodes:
+        ks = sum(n * k for n, k in zip(ep.n_tok(), ep.k(wl.G)))
+        f += 2 * ep.n_query * ep.n_cache * d + 2 * ep.n_query * H * ks * ds + 2 * ep.n_query * H * wl.dh ** 2
+    return f * wl.L
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            j = json.load(f)
+        return {"hbm_gbs": j["hbm_gbs"], "bf16_tflops": j["bf16_tflops"],
+                "bf16_tflops_sustained": j.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def load_traffic(kernel, workload):
+    """DRAM bytes per launch from a committed ncu summary, if it is current.
+
+    profiles/traffic.txt lines: kernel workload source_sha256 dram_bytes
+    """
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    src = os.path.join(ROOT, "paper_2608_18410_gb300", "csrc", kernel + ".cu")
+    if not os.path.exists(src):
+        return None
+    sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    for line in open(path):
+        parts = line.split("#")[0].split()
+        if len(parts) == 4 and parts[0] == kernel and parts[1] == workload and parts[2] == sha:
+            return float(parts[3])
+    return None
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1].split()[0]))
+                mx.append(float(f[2].split()[0]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# distributed helpers (one process per GPU; timing reduce only)
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def max_over_ranks(x, ws):
+    if ws == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(ws):
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# CPU baseline: the oracle on a bounded sample
+# ---------------------------------------------------------------------------
+
+def oracle_sample(wl, inp, budget_s=12.0, max_items=None):
+    """Times the fp64 oracle (compress + attend) on (layer, episode) items of
+    the workload until about budget_s seconds; returns the measurement."""
+    import oracle
+    from paper_2608_18410_gb300 import synth
+    G, H, dh = wl.G, wl.H, wl.dh
+    order = [(l, e) for l in range(wl.L) for e in range(wl.E)]
+    rng = np.random.default_rng(12345)
+    rng.shuffle(order)
+    glob_rows = np.concatenate([[0], np.cumsum([ep.n_cache for ep in wl.episodes])])
+    glob_q = np.concatenate([[0], np.cumsum([ep.n_query for ep in wl.episodes])])
+    items, qtok, t_total = 0, 0, 0.0
+    for (l, e) in order:
+        ep = wl.episodes[e]
+        spec = oracle.Spec(H, dh, G, wl.C, wl.F, np.array(ep.n_tok())[None], np.array(ep.k(G))[None],
+                           [ep.n_query])
+        r0, r1 = int(glob_rows[e]), int(glob_rows[e + 1])
+        q0, q1 = int(glob_q[e]), int(glob_q[e + 1])
+        W = lambda n: synth.widen(inp[n][l], wl.dtype)
+        h = synth.widen(inp["h"][l, r0:r1], wl.dtype)
+        v = synth.widen(inp["v"][l, r0:r1], wl.dtype)
+        q = synth.widen(inp["q"][l, q0:q1], wl.dtype)
+        K = synth.widen(inp["K"][l, r0:r1], wl.dtype)
+        R = W("R")
+        args = (R, W("W_re"), inp["b_re"][l].astype(np.float64), W("W1"), inp["b1"][l].astype(np.float64),
+                W("W2"), inp["b2"][l].astype(np.float64), wl.alpha_role, wl.alpha_lang)
+        t0 = time.perf_counter()
+        c = oracle.compress_layer(spec, h, v, *args, want_z=False)
+        oracle.attend_layer(spec, q, K, c["packed"], c["idx"], R)
+        t_total += time.perf_counter() - t0
+        items += 1
+        qtok += ep.n_query
+        if t_total >= budget_s or (max_items and items >= max_items):
+            break
+    return {"value": qtok / t_total, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{items} (layer, episode) item(s) of {wl.name} ({qtok} query tokens x 1 layer each), "
+                      f"fp64 compress+attend, {t_total:.1f} s, 1 thread"}
+
+
+def run_reference(args):
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    from paper_2608_18410_gb300 import synth
+    wl = make_workload(args.workload)
+    # inputs of a bounded slice: the first layers are enough for the sample
+    inp = synth.gen_inputs(wl.with_layers(min(wl.L, 2)))
+    wl_s = wl.with_layers(min(wl.L, 2))
+    per_step_budget = max(1.0, min(15.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        oracle_sample(wl_s, inp, budget_s=per_step_budget, max_items=1)
+    vals = []
+    meas = None
+    for _ in range(args.steps):
+        meas = oracle_sample(wl_s, inp, budget_s=per_step_budget)
+        vals.append(meas["value"])
+    value = statistics.median(vals)
+    meas["value"] = value
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": None,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": workload_config(wl, flush=None),
+            "cpu_baseline": meas,
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def workload_config(wl, flush):
+    eps = wl.episodes
+    cfg = {"workload": wl.name, "describe": wl.describe, "layers": wl.L, "episodes": wl.E,
+           "heads": wl.H, "head_dim": wl.dh, "groups": wl.G, "role_dim": wl.C, "router_hidden": wl.F,
+           "cache_tokens_per_layer": wl.rows, "query_tokens_per_layer": wl.q_rows,
+           "routed_tokens_per_layer": sum(n for ep in eps for n, k in zip(ep.n_tok(), ep.k(wl.G)) if 0 < k < wl.G),
+           "global_batch": wl.E, "parallelism": "replicas: independent episodes per GPU"}
+    if flush is not None:
+        cfg["l2"] = flush
+    return cfg
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+def run_ours(args):
+    import torch
+    ws, rank, local = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.device("cuda", torch.cuda.current_device())
+    from paper_2608_18410_gb300 import build as pb
+    if rank == 0:
+        pb.build()
+    barrier(ws)
+    from paper_2608_18410_gb300 import rolesub, synth
+
+    wl = make_workload(args.workload, rank)
+    inp = synth.gen_inputs(wl)
+    rs = rolesub.RoleSub(wl.L, wl.H, wl.dh, wl.G, wl.C, wl.F, wl.dtype, wl.n_tok_array(), wl.k_array(),
+                         wl.n_query_array(), device=dev)
+
+    def to_dev(x):
+        t = torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else x)
+        t = t.to(dev)
+        return t.view(torch.bfloat16) if x.dtype == np.uint16 else t
+    d = {k: to_dev(v) for k, v in inp.items()}
+    packed, idx = rs.new_outputs()
+    o = torch.empty((wl.L, max(wl.q_rows, 1), wl.d), dtype=rs.tdtype, device=dev)
+    stream = torch.cuda.current_stream()
+    big = wl.rows * wl.d * 2 * 3 * wl.L > 2 * (129 << 20)
+    flush_buf = None if big else torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def compress():
+        rs.compress(d["h"], d["v"], d["R"], d["W_re"], d["b_re"], d["W1"], d["b1"], d["W2"], d["b2"],
+                    wl.alpha_role, wl.alpha_lang, packed=packed, idx=idx)
+
+    def attend():
+        rs.attend(d["q"], d["K"], packed, idx, d["R"], o=o)
+
+    for _ in range(max(args.warmup, 3)):
+        compress()
+        attend()
+    torch.cuda.synchronize()
+    code, _ = rs.device_status()
+    assert code == 0, f"device status {code}"
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier(ws)
+    torch.cuda.synchronize()
+    launches0 = rolesub.rolesub_launch_count()
+    with ClockSampler(torch.cuda.current_device()) as clk:
+        for i in range(args.steps):
+            if flush_buf is not None:
+                flush_buf.fill_(i & 0xFF)
+            ev[i][0].record(stream)
+            compress()
+            ev[i][1].record(stream)
+            attend()
+            ev[i][2].record(stream)
+        torch.cuda.synchronize()
+    launches = rolesub.rolesub_launch_count() - launches0
+    barrier(ws)
+    t_comp = [a.elapsed_time(b) for a, b, c in ev]
+    t_att = [b.elapsed_time(c) for a, b, c in ev]
+    t_step = [x + y for x, y in zip(t_comp, t_att)]
+    total_ms = max_over_ranks(sum(t_step), ws)
+    ms_per_step = total_ms / args.steps
+    qtok = wl.q_rows * wl.L
+    value = qtok * ws / (ms_per_step / 1e3)
+
+    # ---- end to end through the public API from pinned host buffers --------
+    act = ("h", "v", "K", "q")
+    host = {}
+    for k in act:
+        x = inp[k]
+        t = torch.from_numpy(x.view(np.int16) if x.dtype == np.uint16 else x).pin_memory()
+        host[k] = t
+    o_host = torch.empty(o.shape, dtype=torch.int16 if o.dtype == torch.bfloat16 else o.dtype).pin_memory()
+    h2d = sum(host[k].numel() * host[k].element_size() for k in act)
+    d2h = o_host.numel() * o_host.element_size()
+    dv = {k: (d[k].view(torch.int16) if d[k].dtype == torch.bfloat16 else d[k]) for k in act}
+    ov = o.view(torch.int16) if o.dtype == torch.bfloat16 else o
+
+    def e2e_step():
+        for k in act:
+            dv[k].copy_(host[k], non_blocking=True)
+        compress()
+        attend()
+        o_host.copy_(ov, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e2e_steps = max(1, min(args.steps, 20))
+    barrier(ws)
+    e0.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), ws) / e2e_steps
+    e2e_value = qtok * ws / (e2e_ms / 1e3)
+
+    # ---- roofline of the dominant kernel --------------------------------
+    peaks = load_peaks()
+    att_ms = statistics.mean(t_att)
+    comp_ms = statistics.mean(t_comp)
+    ab = attend_bytes(wl)
+    cb = compress_bytes(wl)
+    att_gbs = ab / (att_ms / 1e3) / 1e9
+    roof = {"kernel": "k_attend (rolesub_attend, one launch per call)", "bound": "hbm",
+            "achieved": att_gbs, "peak": peaks["hbm_gbs"], "unit": "GB/s",
+            "frac": att_gbs / peaks["hbm_gbs"], "peak_source": peaks["source"] + " hbm_gbs (copy)",
+            "algorithmic_bytes_per_launch": ab, "avg_launch_ms": att_ms,
+            "traffic": load_traffic("attend", wl.name),
+            "frac_of_8TBs": att_gbs / 8000.0,
+            "tensor_tflops": attend_flops(wl) / (att_ms / 1e3) / 1e12}
+    comp = {"ms": comp_ms, "algorithmic_bytes": cb, "GB/s": cb / (comp_ms / 1e3) / 1e9,
+            "frac": cb / (comp_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
+
+    clocks = clk.summary()
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+            "config": workload_config(wl, "flushed between steps (512 MB write)" if flush_buf is not None
+                                      else "inputs larger than L2"),
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                    "ms_per_step": e2e_ms},
+            "gpu_launches": launches,
+            "roofline": roof, "compress": comp,
+            "clocks": {"sm_mhz": clocks["sm_mhz"], "sm_max_mhz": clocks["sm_max_mhz"],
+                       "reasons": clocks["reasons"], "samples": clocks["samples"]}}
+    if ws == 1 and rank == 0 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = oracle_sample(wl, inp, budget_s=args.cpu_budget)
+    if rank == 0:
+        print(json.dumps(line))
+    if ws > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default=os.environ.get("ROLESUB_BENCH_WORKLOAD", "c4"),
+                    choices=["c1", "c2", "c3", "c4"])
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args(argv)
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -28,7 +28,8 @@
  *    asynchronous; no entry point synchronises except
  *    rolesub_get_device_status.
  *  - The caller owns every buffer. The library allocates no memory and keeps
- *    no state between calls (one-time per-process lookups aside).
+ *    no state between calls, apart from one-time per-process lookups and a
+ *    diagnostic counter of kernel launches (rolesub_launch_count).
  *  - Device pointers must be 16-byte aligned; ROLESUB_EINVAL otherwise.
  *  - Argument errors return ROLESUB_EINVAL (or ROLESUB_EUNSUPPORTED for a
  *    valid geometry this build does not implement) before anything is
@@ -223,6 +224,11 @@ const char *rolesub_status_string(rolesub_status s);
 
 /* ROLESUB_VERSION of the library actually loaded. */
 int32_t rolesub_version(void);
+
+/* Number of kernels this process has launched through the library so far
+ * (all threads, all devices). Diagnostic only: a caller takes the
+ * difference around a region to count its launches. */
+uint64_t rolesub_launch_count(void);
 
 #ifdef __cplusplus
 }

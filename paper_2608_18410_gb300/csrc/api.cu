@@ -3,10 +3,15 @@
 #include <math.h>
 #include <string.h>
 
-#include <vector>
+#include <atomic>
 
 #include "common.cuh"
 #include "internal.h"
+
+namespace rs {
+static std::atomic<uint64_t> g_launches{0};
+void count_launches(int n) { g_launches.fetch_add((uint64_t)n, std::memory_order_relaxed); }
+}  // namespace rs
 
 namespace {
 
@@ -117,6 +122,8 @@ rolesub_status from_cuda(cudaError_t e) { return e == cudaSuccess ? ROLESUB_OK :
 extern "C" {
 
 int32_t rolesub_version(void) { return ROLESUB_VERSION; }
+
+uint64_t rolesub_launch_count(void) { return rs::g_launches.load(std::memory_order_relaxed); }
 
 const char *rolesub_status_string(rolesub_status s)
 {

@@ -182,6 +182,7 @@ static cudaError_t launch_attend_t(const AttendArgs &a)
         (const T *)a.packed, P.packed_elems_per_layer, a.idx, P.idx_bytes_per_layer,
         (const T *)a.R, pd, S.num_heads, S.num_groups, qtiles, P.q_rows_per_layer, scale,
         (T *)a.o, a.ws.status);
+    count_launches(1);
     return cudaGetLastError();
 }
 

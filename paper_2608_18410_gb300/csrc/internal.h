@@ -60,6 +60,9 @@ cudaError_t launch_rotate_pack(const CompressArgs &a);
 // Routed attention.
 cudaError_t launch_attend(const AttendArgs &a);
 
+// Adds n to the process-wide launch counter (rolesub_launch_count).
+void count_launches(int n);
+
 // Limits of this build (checked before any launch).
 bool router_supported(const rolesub_shape *s);
 bool rotate_supported(const rolesub_shape *s);

@@ -88,6 +88,7 @@ static cudaError_t launch_rot_t(const CompressArgs &a)
                                      S.num_layers), 256, smem, a.stream>>>(
         (const T *)a.v, (const T *)a.R, pd, Ms, P.rows_per_layer, S.num_heads, S.num_groups,
         (T *)a.packed, P.packed_elems_per_layer, a.idx, P.idx_bytes_per_layer, a.ws.status);
+    count_launches(1);
     return cudaGetLastError();
 }
 

@@ -210,6 +210,7 @@ static cudaError_t launch_router_t(const CompressArgs &a)
     k_router_epilogue<T><<<dim3((unsigned)((M + 7) / 8), L), 256, smem, a.stream>>>(
         a.ws.logits, pd, M, d, C, F, G, E, W1, a.ws.lang_bias, W2, a.b2, a.alpha_role, a.idx,
         P.idx_bytes_per_layer);
+    count_launches(4);
     return cudaGetLastError();
 }
 

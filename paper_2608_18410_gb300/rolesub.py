@@ -29,7 +29,8 @@ STATUS = {0: "ROLESUB_OK", 1: "ROLESUB_EINVAL", 2: "ROLESUB_EUNSUPPORTED", 3: "R
 # every symbol include/rolesub.h declares
 EXPORTS = ("rolesub_plan_size", "rolesub_layout_plan", "rolesub_workspace_size",
            "rolesub_compress", "rolesub_attend", "rolesub_get_device_status",
-           "rolesub_reset_device_status", "rolesub_status_string", "rolesub_version")
+           "rolesub_reset_device_status", "rolesub_status_string", "rolesub_version",
+           "rolesub_launch_count")
 
 
 class RoleSubError(RuntimeError):
@@ -101,8 +102,10 @@ def lib():
         L.rolesub_status_string.restype = ctypes.c_char_p
         L.rolesub_version.argtypes = []
         L.rolesub_version.restype = ctypes.c_int32
+        L.rolesub_launch_count.argtypes = []
+        L.rolesub_launch_count.restype = ctypes.c_uint64
         for name in EXPORTS:
-            if name not in ("rolesub_status_string", "rolesub_version"):
+            if name not in ("rolesub_status_string", "rolesub_version", "rolesub_launch_count"):
                 getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -222,6 +225,10 @@ def rolesub_status_string(code):
 
 def rolesub_version():
     return int(lib().rolesub_version())
+
+
+def rolesub_launch_count():
+    return int(lib().rolesub_launch_count())
 
 
 # ---------------------------------------------------------------------------
