@@ -62,7 +62,8 @@ typedef enum {
     ROLESUB_EUNSUPPORTED = 2,  /* geometry not implemented; nothing launched  */
     ROLESUB_ECUDA = 3,         /* CUDA runtime error or failed launch         */
     ROLESUB_EDEVICE = 4,       /* kernel found bad data (device status word)  */
-    ROLESUB_ETIMEOUT = 5       /* a bounded in-kernel wait gave up            */
+    ROLESUB_ETIMEOUT = 5,      /* a bounded in-kernel wait gave up            */
+    ROLESUB_ETOOLARGE = 6      /* needs more than the static scratch holds    */
 } rolesub_status;
 
 typedef enum { ROLESUB_F32 = 0, ROLESUB_BF16 = 1 } rolesub_dtype;
@@ -224,6 +225,44 @@ const char *rolesub_status_string(rolesub_status s);
 
 /* ROLESUB_VERSION of the library actually loaded. */
 int32_t rolesub_version(void);
+
+/*
+ * rolesub_compress_static -- rolesub_compress for callers that cannot
+ * allocate device memory. (The paper has no counterpart: this is a
+ * deployment variant of the compress call.)
+ *
+ * Some callers cannot call cudaMalloc at the point where they compress: a
+ * serving engine or robot-control loop that reserves all of its device
+ * memory up front and forbids allocation afterwards, or a plug-in whose
+ * host framework hands it inputs and outputs but no scratch buffer. This
+ * entry point takes the same inputs and outputs as rolesub_compress, minus
+ * the workspace: its scratch (language contexts, per-episode biases,
+ * router logits, status word) lives in a fixed array compiled into the
+ * library, ROLESUB_STATIC_SCRATCH_BYTES per GPU, which every GPU that loads
+ * the library holds until the process exits. It calls no allocator.
+ *
+ * Limits and behaviour:
+ *  - Problems whose scratch (rolesub_workspace_size) exceeds
+ *    ROLESUB_STATIC_SCRATCH_BYTES return ROLESUB_ETOOLARGE; nothing runs.
+ *  - The first call on a device looks up the array's device address (once
+ *    per device, with that device current); make that first call before
+ *    any stream capture.
+ *  - Every call shares the one array and leaves its contents behind; the
+ *    call clears what must start at zero itself. Calls whose work overlaps
+ *    on the GPU (different streams, or different host threads on one
+ *    device) race on the array: serialise them.
+ *  - The device status word is kept in the array and is not readable by
+ *    the caller; the compress kernels only report stored indices >= S,
+ *    which the router does not produce.
+ * Other arguments, errors and results: as rolesub_compress.
+ */
+#define ROLESUB_STATIC_SCRATCH_BYTES (8u << 20)
+rolesub_status rolesub_compress_static(const rolesub_shape *shape, const void *plan_host,
+                                       const void *plan_dev, const void *h, const void *v,
+                                       const void *R, const void *W_re, const float *b_re,
+                                       const void *W1, const float *b1, const void *W2,
+                                       const float *b2, float alpha_role, float alpha_lang,
+                                       void *packed_v, uint8_t *idx, void *stream);
 
 /* Number of kernels this process has launched through the library so far
  * (all threads, all devices). Diagnostic only: a caller takes the

@@ -134,6 +134,7 @@ const char *rolesub_status_string(rolesub_status s)
     case ROLESUB_ECUDA: return "CUDA error";
     case ROLESUB_EDEVICE: return "bad data found on the device";
     case ROLESUB_ETIMEOUT: return "in-kernel wait timed out";
+    case ROLESUB_ETOOLARGE: return "problem needs more scratch than the library's static array";
     }
     return "unknown status";
 }
@@ -364,3 +365,88 @@ rolesub_status rolesub_reset_device_status(void *workspace, void *stream)
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// rolesub_compress_static: compress without any allocation by the caller or
+// the library. Its scratch is this fixed array, one per GPU that loads the
+// library, held until the process exits. The host only ever passes the
+// array's device address, looked up once per device; host code never
+// dereferences the symbol itself (on the host it names a stand-in, not
+// device memory).
+// ---------------------------------------------------------------------------
+#include <mutex>
+
+static __device__ __align__(256) unsigned char g_compress_scratch[ROLESUB_STATIC_SCRATCH_BYTES];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_scratch_mu;
+void *g_scratch_addr[kMaxDevices];  // device address of g_compress_scratch per device
+
+// Device address of the scratch array on the current device (set-up on the
+// first call per device).
+rolesub_status static_scratch(void **out)
+{
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return ROLESUB_ECUDA;
+    std::lock_guard<std::mutex> lk(g_scratch_mu);
+    if (!g_scratch_addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_compress_scratch) != cudaSuccess || !p) return ROLESUB_ECUDA;
+        g_scratch_addr[dev] = p;
+    }
+    *out = g_scratch_addr[dev];
+    return ROLESUB_OK;
+}
+
+}  // namespace
+
+extern "C" rolesub_status rolesub_compress_static(
+    const rolesub_shape *shape, const void *plan_host, const void *plan_dev, const void *h,
+    const void *v, const void *R, const void *W_re, const float *b_re, const void *W1,
+    const float *b1, const void *W2, const float *b2, float alpha_role, float alpha_lang,
+    void *packed_v, uint8_t *idx, void *stream)
+{
+    if (!shape_ok(shape)) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, plan_dev, &pv);
+    if (st != ROLESUB_OK) return st;
+    if (!plan_dev) return ROLESUB_EINVAL;
+    const void *ptrs[] = {h, v, R, W_re, b_re, W1, b1, W2, b2};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    const rolesub_plan &P = *pv.hdr;
+    if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
+    if (P.idx_bytes_per_layer > 0 && (!idx || !aligned16(idx))) return ROLESUB_EINVAL;
+    if (!isfinite(alpha_role) || !isfinite(alpha_lang)) return ROLESUB_EINVAL;
+    const WsSizes w = ws_sizes(shape, pv.hdr);
+    if (w.total > (size_t)ROLESUB_STATIC_SCRATCH_BYTES) return ROLESUB_ETOOLARGE;
+    if (!rs::router_supported(shape) || !rs::rotate_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    void *scratch = nullptr;
+    st = static_scratch(&scratch);
+    if (st != ROLESUB_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    // the previous call's status word is still in the array
+    if (cudaMemsetAsync(scratch, 0, rs::kStatusBytes, s) != cudaSuccess) return ROLESUB_ECUDA;
+    rs::CompressArgs a;
+    a.shape = shape;
+    a.plan = pv;
+    a.ws = carve(w, scratch);
+    a.h = h;
+    a.v = v;
+    a.R = R;
+    a.W_re = W_re;
+    a.W1 = W1;
+    a.W2 = W2;
+    a.b_re = b_re;
+    a.b1 = b1;
+    a.b2 = b2;
+    a.alpha_role = alpha_role;
+    a.alpha_lang = alpha_lang;
+    a.packed = packed_v;
+    a.idx = idx;
+    a.stream = s;
+    if (rs::launch_router(a) != cudaSuccess) return ROLESUB_ECUDA;
+    return from_cuda(rs::launch_rotate_pack(a));
+}

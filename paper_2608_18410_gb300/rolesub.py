@@ -24,13 +24,15 @@ NUM_KINDS = 4
 PLAN_MAGIC = 0x42555352
 
 STATUS = {0: "ROLESUB_OK", 1: "ROLESUB_EINVAL", 2: "ROLESUB_EUNSUPPORTED", 3: "ROLESUB_ECUDA",
-          4: "ROLESUB_EDEVICE", 5: "ROLESUB_ETIMEOUT"}
+          4: "ROLESUB_EDEVICE", 5: "ROLESUB_ETIMEOUT", 6: "ROLESUB_ETOOLARGE"}
 
 # every symbol include/rolesub.h declares
 EXPORTS = ("rolesub_plan_size", "rolesub_layout_plan", "rolesub_workspace_size",
            "rolesub_compress", "rolesub_attend", "rolesub_get_device_status",
            "rolesub_reset_device_status", "rolesub_status_string", "rolesub_version",
-           "rolesub_launch_count")
+           "rolesub_launch_count", "rolesub_compress_static")
+
+STATIC_SCRATCH_BYTES = 8 << 20
 
 
 class RoleSubError(RuntimeError):
@@ -102,6 +104,8 @@ def lib():
         L.rolesub_status_string.restype = ctypes.c_char_p
         L.rolesub_version.argtypes = []
         L.rolesub_version.restype = ctypes.c_int32
+        L.rolesub_compress_static.argtypes = ([sp, _vp, _vp] + [_vp] * 9 + [ctypes.c_float, ctypes.c_float]
+                                              + [_vp, _vp, _vp])
         L.rolesub_launch_count.argtypes = []
         L.rolesub_launch_count.restype = ctypes.c_uint64
         for name in EXPORTS:
@@ -205,6 +209,16 @@ def rolesub_attend(shape, plan: Plan, plan_dev, q, q_strides, K, k_strides, pack
         ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(q), *[int(s) for s in q_strides],
         _ptr(K), *[int(s) for s in k_strides], _ptr(packed_v), _ptr(idx), _ptr(R),
         float(softmax_scale), _ptr(o), _ptr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def rolesub_compress_static(shape, plan: Plan, plan_dev, h, v, R, W_re, b_re, W1, b1, W2, b2,
+                            alpha_role, alpha_lang, packed_v, idx, stream=None):
+    """rolesub_compress for callers that cannot allocate: the scratch is the
+    library's fixed per-GPU array (STATIC_SCRATCH_BYTES); no workspace."""
+    _check("rolesub_compress_static", lib().rolesub_compress_static(
+        ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(h), _ptr(v), _ptr(R), _ptr(W_re),
+        _ptr(b_re), _ptr(W1), _ptr(b1), _ptr(W2), _ptr(b2), float(alpha_role), float(alpha_lang),
+        _ptr(packed_v), _ptr(idx), _stream(stream)))
 
 
 def rolesub_get_device_status(workspace, stream=None):
