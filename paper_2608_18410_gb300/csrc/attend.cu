@@ -188,6 +188,7 @@ static cudaError_t launch_attend_t(const AttendArgs &a)
 
 cudaError_t launch_attend(const AttendArgs &a)
 {
+    if (attend_tc_supported(a.shape)) return launch_attend_tc(a);
     const bool bf = a.shape->dtype == ROLESUB_BF16;
     if (a.shape->head_dim == 128)
         return bf ? launch_attend_t<__nv_bfloat16, 128>(a) : launch_attend_t<float, 128>(a);

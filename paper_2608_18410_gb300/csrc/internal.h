@@ -59,6 +59,9 @@ cudaError_t launch_router(const CompressArgs &a);
 cudaError_t launch_rotate_pack(const CompressArgs &a);
 // Routed attention.
 cudaError_t launch_attend(const AttendArgs &a);
+// Routed attention on tcgen05/TMA (bf16, d_h = 128, S = 16).
+bool attend_tc_supported(const rolesub_shape *s);
+cudaError_t launch_attend_tc(const AttendArgs &a);
 
 // Adds n to the process-wide launch counter (rolesub_launch_count).
 void count_launches(int n);
