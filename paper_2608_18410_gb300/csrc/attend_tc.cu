@@ -25,7 +25,6 @@
 // region and only produce output rows that are never read.
 // TMEM (256 columns): S buffers at 0 and 64, Y_c at 128, O at 0.
 #include <cuda.h>
-#include <cudaTypedefs.h>
 
 #include "common.cuh"
 #include "internal.h"
@@ -356,40 +355,6 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
     }
 }
 
-// -------------------------------------------------------------- host side
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
-{
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = [] {
-        void *p = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
-                cudaSuccess ||
-            q != cudaDriverEntryPointSuccess)
-            return (PFN_cuTensorMapEncodeTiled_v12000) nullptr;
-        return (PFN_cuTensorMapEncodeTiled_v12000)p;
-    }();
-    return fn;
-}
-
-// bf16 tensor map with 128-byte swizzle; dims/strides innermost first.
-bool make_map(CUtensorMap *m, const void *base, int rank, const uint64_t *dims, const uint64_t *strides_bytes,
-              const uint32_t *box)
-{
-    auto fn = encode_fn();
-    if (!fn) return false;
-    cuuint64_t gd[5], gs[4];
-    cuuint32_t bx[5], es[5];
-    for (int i = 0; i < rank; ++i) {
-        gd[i] = dims[i];
-        bx[i] = box[i];
-        es[i] = 1;
-        if (i + 1 < rank) gs[i] = strides_bytes[i];
-    }
-    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void *>(base), gd, gs, bx, es,
-              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 }  // namespace
 
 bool attend_tc_supported(const rolesub_shape *s)
@@ -408,19 +373,19 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
         const uint64_t dims[4] = {(uint64_t)kDh, (uint64_t)H, (uint64_t)P.q_rows_per_layer, (uint64_t)L};
         const uint64_t str[3] = {(uint64_t)a.q_hs * 2, (uint64_t)a.q_rs * 2, (uint64_t)a.q_ls * 2};
         const uint32_t box[4] = {64, 1, (uint32_t)kQRows, 1};
-        if (!make_map(&tq, a.q, 4, dims, str, box)) return cudaErrorInvalidValue;
+        if (!make_bf16_map(&tq, a.q, 4, dims, str, box)) return cudaErrorInvalidValue;
     }
     {
         const uint64_t dims[4] = {(uint64_t)kDh, (uint64_t)H, (uint64_t)P.rows_per_layer, (uint64_t)L};
         const uint64_t str[3] = {(uint64_t)a.k_hs * 2, (uint64_t)a.k_rs * 2, (uint64_t)a.k_ls * 2};
         const uint32_t box[4] = {64, 1, (uint32_t)kChunk, 1};
-        if (!make_map(&tk, a.K, 4, dims, str, box)) return cudaErrorInvalidValue;
+        if (!make_bf16_map(&tk, a.K, 4, dims, str, box)) return cudaErrorInvalidValue;
     }
     {
         const uint64_t dims[3] = {(uint64_t)kDh, (uint64_t)kDh, (uint64_t)L * H};
         const uint64_t str[2] = {(uint64_t)kDh * 2, (uint64_t)kDh * kDh * 2};
         const uint32_t box[3] = {64, (uint32_t)kDh, 1};
-        if (!make_map(&tr, a.R, 3, dims, str, box)) return cudaErrorInvalidValue;
+        if (!make_bf16_map(&tr, a.R, 3, dims, str, box)) return cudaErrorInvalidValue;
     }
     cudaError_t err = cudaFuncSetAttribute(k_attend_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (err != cudaSuccess) return err;

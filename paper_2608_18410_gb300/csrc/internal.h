@@ -7,6 +7,8 @@
 
 #include "rolesub.h"
 
+struct CUtensorMap_st;
+
 namespace rs {
 
 struct PlanView {  // host view of a validated plan + device copy
@@ -57,6 +59,9 @@ struct AttendArgs {
 cudaError_t launch_router(const CompressArgs &a);
 // Rotation z = R_h^T v and packing of the kept groups.
 cudaError_t launch_rotate_pack(const CompressArgs &a);
+// Rotation and packing on tcgen05/TMA (bf16, d_h = 128, S = 16).
+bool rotate_tc_supported(const rolesub_shape *s);
+cudaError_t launch_rotate_tc(const CompressArgs &a);
 // Routed attention.
 cudaError_t launch_attend(const AttendArgs &a);
 // Routed attention on tcgen05/TMA (bf16, d_h = 128, S = 16).
@@ -65,6 +70,10 @@ cudaError_t launch_attend_tc(const AttendArgs &a);
 
 // Adds n to the process-wide launch counter (rolesub_launch_count).
 void count_launches(int n);
+
+// bf16 TMA descriptor with 128-byte swizzle (dims and strides innermost first).
+bool make_bf16_map(CUtensorMap_st *m, const void *base, int rank, const uint64_t *dims,
+                   const uint64_t *strides_bytes, const uint32_t *box);
 
 // Limits of this build (checked before any launch).
 bool router_supported(const rolesub_shape *s);

@@ -94,6 +94,7 @@ static cudaError_t launch_rot_t(const CompressArgs &a)
 
 cudaError_t launch_rotate_pack(const CompressArgs &a)
 {
+    if (rotate_tc_supported(a.shape)) return launch_rotate_tc(a);
     const bool bf = a.shape->dtype == ROLESUB_BF16;
     if (a.shape->head_dim == 128)
         return bf ? launch_rot_t<__nv_bfloat16, 128>(a) : launch_rot_t<float, 128>(a);
