@@ -129,6 +129,9 @@ typedef struct {
     int64_t off_routed_rows;         /* int32[routed_rows]: ascending row ids  */
     int64_t off_stored_rows;         /* int32[stored_rows]: ascending row ids  */
     int64_t total_bytes;             /* size of the whole blob                 */
+    int32_t num_route_tiles;         /* 128-row windows covering routed rows   */
+    int32_t reserved2;
+    int64_t off_route_tiles;         /* int32[num_route_tiles]: first row      */
 } rolesub_plan;
 
 /* Bytes needed for the plan of num_episodes episodes with n_tok[e*4+kind]

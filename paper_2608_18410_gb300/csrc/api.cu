@@ -40,7 +40,7 @@ bool shape_ok(const rolesub_shape *s)
 }
 
 struct Sizes {
-    size_t header, segs, eps, row_seg, routed, stored, total;
+    size_t header, segs, eps, row_seg, routed, stored, tiles, total;
 };
 
 Sizes plan_sizes(int32_t E, int64_t rows)
@@ -52,7 +52,8 @@ Sizes plan_sizes(int32_t E, int64_t rows)
     z.row_seg = align_up(sizeof(int32_t) * (size_t)rows, 16);
     z.routed = z.row_seg;
     z.stored = z.row_seg;
-    z.total = z.header + z.segs + z.eps + z.row_seg + z.routed + z.stored;
+    z.tiles = z.row_seg;   // at most one router tile per routed row
+    z.total = z.header + z.segs + z.eps + z.row_seg + z.routed + z.stored + z.tiles;
     return z;
 }
 
@@ -81,6 +82,7 @@ rolesub_status view_plan(const rolesub_shape *s, const void *plan_host, const vo
     pv->row_seg_dev = d ? (const int32_t *)(d + p->off_row_seg) : nullptr;
     pv->routed_dev = d ? (const int32_t *)(d + p->off_routed_rows) : nullptr;
     pv->stored_dev = d ? (const int32_t *)(d + p->off_stored_rows) : nullptr;
+    pv->route_tiles_dev = d ? (const int32_t *)(d + p->off_route_tiles) : nullptr;
     return ROLESUB_OK;
 }
 
@@ -96,9 +98,13 @@ WsSizes ws_sizes(const rolesub_shape *s, const rolesub_plan *p)
     w.status = rs::kStatusBytes;
     w.ctx = align_up(sizeof(float) * L * E * d, kAlign);
     w.bias = align_up(sizeof(float) * L * E * s->router_hidden, kAlign);
-    w.logits = align_up(sizeof(float) * L * (size_t)p->routed_rows_per_layer *
-                            (size_t)(s->router_hidden + s->role_dim),
-                        kAlign);
+    // router logits are only staged in memory when the fused tensor-core
+    // router does not apply
+    w.logits = rs::router_tc_supported(s)
+                   ? 0
+                   : align_up(sizeof(float) * L * (size_t)p->routed_rows_per_layer *
+                                  (size_t)(s->router_hidden + s->role_dim),
+                              kAlign);
     w.total = w.status + w.ctx + w.bias + w.logits;
     return w;
 }
@@ -185,6 +191,7 @@ rolesub_status rolesub_layout_plan(const rolesub_shape *shape, int32_t E, const 
     p->off_row_seg = (int64_t)(z.header + z.segs + z.eps);
     p->off_routed_rows = p->off_row_seg + (int64_t)z.row_seg;
     p->off_stored_rows = p->off_routed_rows + (int64_t)z.routed;
+    p->off_route_tiles = p->off_stored_rows + (int64_t)z.stored;
     p->total_bytes = (int64_t)z.total;
     rolesub_segment *segs = (rolesub_segment *)(b + p->off_segments);
     rolesub_episode *eps = (rolesub_episode *)(b + p->off_episodes);
@@ -237,6 +244,18 @@ rolesub_status rolesub_layout_plan(const rolesub_shape *shape, int32_t E, const 
     p->stored_rows_per_layer = nstored;
     p->max_cache_tokens = max_c;
     p->max_query_tokens = max_q;
+    // router tiles: 128-row windows, each starting at the first routed row
+    // the previous windows left uncovered
+    int32_t *tiles = (int32_t *)(b + p->off_route_tiles);
+    int32_t nt = 0;
+    int64_t covered = -1;
+    for (int64_t i = 0; i < nrouted; ++i) {
+        if (routed[i] > covered) {
+            tiles[nt++] = routed[i];
+            covered = (int64_t)routed[i] + 127;
+        }
+    }
+    p->num_route_tiles = nt;
     return ROLESUB_OK;
 }
 

@@ -48,6 +48,7 @@ struct PlanDev {
     const int32_t *row_seg;
     const int32_t *routed;
     const int32_t *stored;
+    const int32_t *route_tiles;
 };
 
 }  // namespace rs

@@ -21,6 +21,7 @@ struct PlanView {  // host view of a validated plan + device copy
     const int32_t *row_seg_dev;
     const int32_t *routed_dev;
     const int32_t *stored_dev;
+    const int32_t *route_tiles_dev;
 };
 
 struct Workspace {  // carve-up of the caller's workspace
@@ -59,6 +60,10 @@ struct AttendArgs {
 cudaError_t launch_router(const CompressArgs &a);
 // Rotation z = R_h^T v and packing of the kept groups.
 cudaError_t launch_rotate_pack(const CompressArgs &a);
+// Fused router GEMM + epilogue + top-k on tcgen05/TMA (bf16, F = 256,
+// C = 64, S = 16); needs the per-episode biases in the workspace.
+bool router_tc_supported(const rolesub_shape *s);
+cudaError_t launch_router_tc(const CompressArgs &a);
 // Rotation and packing on tcgen05/TMA (bf16, d_h = 128, S = 16).
 bool rotate_tc_supported(const rolesub_shape *s);
 cudaError_t launch_rotate_tc(const CompressArgs &a);

@@ -202,6 +202,11 @@ static cudaError_t launch_router_t(const CompressArgs &a)
         h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
     k_lang_bias<T><<<dim3((F + 7) / 8, L), 256, 0, a.stream>>>(
         W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+    if (router_tc_supported(a.shape)) {
+        count_launches(2);
+        cudaError_t e = cudaGetLastError();
+        return e != cudaSuccess ? e : launch_router_tc(a);
+    }
     k_router_gemm_simt<T><<<dim3((unsigned)((M + 63) / 64), (F + C + 63) / 64, L), 256, 0, a.stream>>>(
         h, a.plan.routed_dev, M, P.rows_per_layer, d, C, F, W1, Wre, a.b_re, a.ws.logits);
     PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev,

@@ -1,0 +1,346 @@
+// router_tc.cu -- role-conditioned group scores and top-k on the
+// 5th-generation tensor core (Sec. 3.3-3.4), bf16 inputs.
+//
+// One CTA per (128-row router tile, layer), 192 threads:
+//   warp 4  TMA producer, warp 5  MMA issuer, warps 0-3  epilogue (a
+//   thread per tile row / TMEM lane).
+// Mainloop over the hidden size d in 64-column blocks (3-stage TMA ring):
+//   TMEM[0,256)   += h W1_h^T      (first d input columns of W1)
+//   TMEM[256,320) += h W_re^T      (role logits)
+// Epilogue, per routed row i:
+//   a   = softmax(W_re h + b_re)                      Eq. (latentrole)
+//   TMEM[0,256) += (alpha_role a) W1_a^T              tensor core, with
+//         alpha_role a split into bf16 hi + lo parts (two MMAs) so the
+//         product keeps ~16 mantissa bits
+//   u   = ReLU(TMEM[0,256) + beta_e)                  beta_e = W1_c (alpha_lang
+//         c_e) + b1 from the per-episode kernel
+//   gamma = u W2^T + b2                               again hi + lo MMAs
+//   keep the k largest gamma (ties: lower index), indices ascending.
+// The scores that decide the top-k are thus computed with fp32
+// accumulation and near-fp32 operands; no fp32 intermediate is rounded to
+// plain bf16.
+#include <cuda.h>
+
+#include "common.cuh"
+#include "internal.h"
+#include "sm100.cuh"
+
+namespace rs {
+
+namespace {
+
+using namespace sm100;
+typedef __nv_bfloat16 bf16;
+
+constexpr int kThreads = 192;
+constexpr int kRows = 128;
+constexpr int kF = 256;      // router hidden
+constexpr int kC = 64;       // role dim
+constexpr int kG = 16;       // groups
+constexpr int kStages = 3;
+
+constexpr uint32_t kStageBytes = 16384 + 32768 + 8192;       // A | W1_h | W_re
+constexpr uint32_t kOffW1A = kStages * kStageBytes;          // 168K: W1_a [256][64]
+constexpr uint32_t kOffW2 = kOffW1A + 32768;                 // 200K: W2 [16][256]
+constexpr uint32_t kOffBar = kOffW2 + 8192;                  // 208K
+constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
+// epilogue operands reuse the (drained) stage ring
+constexpr uint32_t kOffARhi = 0, kOffARlo = 16384, kOffUhi = 32768, kOffUlo = 98304;
+
+constexpr uint32_t kIdescH = idesc_bf16(128, 256, false);
+constexpr uint32_t kIdescR = idesc_bf16(128, 64, false);
+constexpr uint32_t kIdescG = idesc_bf16(128, 16, false);
+
+__device__ __forceinline__ void split_bf16(float x, float &hi_out, uint16_t &hi, uint16_t &lo)
+{
+    const bf16 h = __float2bfloat16_rn(x);
+    const float hf = __bfloat162float(h);
+    const bf16 l = __float2bfloat16_rn(x - hf);
+    hi = *reinterpret_cast<const uint16_t *>(&h);
+    lo = *reinterpret_cast<const uint16_t *>(&l);
+    hi_out = hf;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_w1,
+            const __grid_constant__ CUtensorMap tm_wre, const __grid_constant__ CUtensorMap tm_w2,
+            PlanDev plan, int64_t rows, int d, int E, int G, const float *__restrict__ b_re,
+            const float *__restrict__ beta, const float *__restrict__ b2, float alpha_role,
+            uint8_t *__restrict__ idx, int64_t idx_per_layer, int32_t *status)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ uint32_t tmem_slot;
+    __shared__ volatile int abort_flag;
+    const uint32_t sraw = smem_u32(smem_raw);
+    const uint32_t sb = (sraw + 1023u) & ~1023u;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int l = blockIdx.y;
+    const int row0 = plan.route_tiles[blockIdx.x];
+    const int nkb = d / 64;
+
+    const uint32_t bar_full = sb + kOffBar;            // [3]
+    const uint32_t bar_empty = bar_full + 24;          // [3]
+    const uint32_t bar_acc = bar_full + 48, bar_w = bar_full + 56, bar_ar = bar_full + 64,
+                   bar_h = bar_full + 72, bar_u = bar_full + 80, bar_g = bar_full + 88;
+
+    if (tid == 0) {
+        abort_flag = 0;
+        for (int i = 0; i < 6; ++i) mbar_init(bar_full + 8 * i, 1);
+        mbar_init(bar_acc, 1);
+        mbar_init(bar_w, 1);
+        mbar_init(bar_ar, 128);
+        mbar_init(bar_h, 1);
+        mbar_init(bar_u, 128);
+        mbar_init(bar_g, 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (warp == 0) {
+        tmem_alloc(smem_u32(&tmem_slot), 512);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+
+    if (warp == 4) {
+        if (lane == 0) {
+            prefetch_tmap(&tm_h);
+            prefetch_tmap(&tm_w1);
+            prefetch_tmap(&tm_wre);
+            prefetch_tmap(&tm_w2);
+            // epilogue weights of this layer: W1_a (input columns d..d+C) and W2
+            mbar_expect_tx(bar_w, 32768 + 8192);
+            tma_load_3d(sb + kOffW1A, &tm_w1, d, 0, l, bar_w);
+            for (int kb = 0; kb < 4; ++kb) tma_load_3d(sb + kOffW2 + 2048 * kb, &tm_w2, 64 * kb, 0, l, bar_w);
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int s = kb % kStages;
+                if (kb >= kStages && !mbar_wait(bar_empty + 8 * s, ((kb / kStages) - 1) & 1, status, &abort_flag, 20))
+                    break;
+                const uint32_t st = sb + kStageBytes * s;
+                mbar_expect_tx(bar_full + 8 * s, kStageBytes);
+                tma_load_3d(st, &tm_h, 64 * kb, row0, l, bar_full + 8 * s);
+                tma_load_3d(st + 16384, &tm_w1, 64 * kb, 0, l, bar_full + 8 * s);
+                tma_load_3d(st + 49152, &tm_wre, 64 * kb, 0, l, bar_full + 8 * s);
+            }
+        }
+    } else if (warp == 5) {
+        if (lane == 0) {
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int s = kb % kStages;
+                if (!mbar_wait(bar_full + 8 * s, (kb / kStages) & 1, status, &abort_flag, 21)) break;
+                tc_fence_after();
+                const uint32_t st = sb + kStageBytes * s;
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) {
+                    const uint64_t a = sdesc_sw128(st + 32u * kk, 16, 1024);
+                    const uint32_t acc = (kb > 0 || kk > 0) ? 1u : 0u;
+                    mma_bf16(tmem, a, sdesc_sw128(st + 16384 + 32u * kk, 16, 1024), kIdescH, acc);
+                    mma_bf16(tmem + 256, a, sdesc_sw128(st + 49152 + 32u * kk, 16, 1024), kIdescR, acc);
+                }
+                mma_commit(bar_empty + 8 * s);
+            }
+            mma_commit(bar_acc);
+            // hidden += (alpha_role a) W1_a^T, hi and lo parts
+            if (mbar_wait(bar_ar, 0, status, &abort_flag, 22) && mbar_wait(bar_w, 0, status, &abort_flag, 23)) {
+                tc_fence_after();
+#pragma unroll
+                for (int part = 0; part < 2; ++part)
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        mma_bf16(tmem, sdesc_sw128(sb + (part ? kOffARlo : kOffARhi) + 32u * kk, 16, 1024),
+                                 sdesc_sw128(sb + kOffW1A + 32u * kk, 16, 1024), kIdescH, 1u);
+            }
+            mma_commit(bar_h);
+            // gamma = u W2^T, hi and lo parts
+            if (mbar_wait(bar_u, 0, status, &abort_flag, 24)) {
+                tc_fence_after();
+#pragma unroll
+                for (int part = 0; part < 2; ++part)
+#pragma unroll
+                    for (int kk = 0; kk < 16; ++kk) {
+                        const uint32_t ao = (part ? kOffUlo : kOffUhi) + (kk >> 2) * 16384u + (kk & 3) * 32u;
+                        const uint32_t bo = kOffW2 + (kk >> 2) * 2048u + (kk & 3) * 32u;
+                        mma_bf16(tmem + 320, sdesc_sw128(sb + ao, 16, 1024), sdesc_sw128(sb + bo, 16, 1024), kIdescG,
+                                 (part > 0 || kk > 0) ? 1u : 0u);
+                    }
+            }
+            mma_commit(bar_g);
+        }
+    } else {
+        // ------------------------------------------------ epilogue warps 0-3
+        const int64_t r = (int64_t)row0 + tid;
+        bool routed = false;
+        rolesub_segment sg{};
+        if (r < rows) {
+            sg = plan.segs[plan.row_seg[r]];
+            routed = sg.k > 0 && sg.k < G;
+        }
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
+        const uint32_t swz = (uint32_t)(tid & 7);
+        mbar_wait(bar_acc, 0, status, &abort_flag, 25);
+        tc_fence_after();
+        __syncwarp();
+        // role softmax -> alpha_role * a, split into bf16 hi / lo operand rows
+        {
+            uint32_t sr[32];
+            float lg[kC];
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                tmem_ld32(lane_base + 256 + 32 * q, sr);
+                tmem_wait_ld();
+#pragma unroll
+                for (int j = 0; j < 32; ++j) lg[32 * q + j] = __uint_as_float(sr[j]) + __ldg(b_re + (int64_t)l * kC + 32 * q + j);
+            }
+            float mx = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < kC; ++c) mx = fmaxf(mx, lg[c]);
+            float sum = 0.f;
+#pragma unroll
+            for (int c = 0; c < kC; ++c) {
+                lg[c] = expf(lg[c] - mx);
+                sum += lg[c];
+            }
+            const float sc = alpha_role / sum;
+#pragma unroll
+            for (int cc = 0; cc < 8; ++cc) {
+                uint32_t hw[4], lw[4];
+#pragma unroll
+                for (int p = 0; p < 4; ++p) {
+                    float dummy;
+                    uint16_t h0, l0, h1, l1;
+                    split_bf16(lg[8 * cc + 2 * p] * sc, dummy, h0, l0);
+                    split_bf16(lg[8 * cc + 2 * p + 1] * sc, dummy, h1, l1);
+                    hw[p] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+                    lw[p] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+                }
+                const uint32_t off = (uint32_t)tid * 128u + (((uint32_t)cc ^ swz) << 4);
+                st_shared_v4(sb + kOffARhi + off, hw[0], hw[1], hw[2], hw[3]);
+                st_shared_v4(sb + kOffARlo + off, lw[0], lw[1], lw[2], lw[3]);
+            }
+        }
+        fence_async_smem();
+        mbar_arrive(bar_ar);
+        // u = ReLU(hidden + beta_e), split into bf16 hi / lo operand rows
+        mbar_wait(bar_h, 0, status, &abort_flag, 26);
+        tc_fence_after();
+        __syncwarp();
+        {
+            const float *be = beta + ((int64_t)l * E + sg.episode) * kF;
+#pragma unroll 1
+            for (int q = 0; q < 8; ++q) {
+                uint32_t sr[32];
+                tmem_ld32(lane_base + 32 * q, sr);
+                tmem_wait_ld();
+#pragma unroll
+                for (int cc = 0; cc < 4; ++cc) {
+                    uint32_t hw[4], lw[4];
+#pragma unroll
+                    for (int p = 0; p < 4; ++p) {
+                        const int j = 8 * cc + 2 * p;
+                        const float u0 = fmaxf(__uint_as_float(sr[j]) + (routed ? __ldg(be + 32 * q + j) : 0.f), 0.f);
+                        const float u1 = fmaxf(__uint_as_float(sr[j + 1]) + (routed ? __ldg(be + 32 * q + j + 1) : 0.f), 0.f);
+                        float dummy;
+                        uint16_t h0, l0, h1, l1;
+                        split_bf16(u0, dummy, h0, l0);
+                        split_bf16(u1, dummy, h1, l1);
+                        hw[p] = (uint32_t)h0 | ((uint32_t)h1 << 16);
+                        lw[p] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+                    }
+                    const int chunk = 4 * q + cc;   // 16-byte chunk of the 256-column row
+                    const uint32_t off = (uint32_t)(chunk >> 3) * 16384u + (uint32_t)tid * 128u +
+                                         (((uint32_t)(chunk & 7) ^ swz) << 4);
+                    st_shared_v4(sb + kOffUhi + off, hw[0], hw[1], hw[2], hw[3]);
+                    st_shared_v4(sb + kOffUlo + off, lw[0], lw[1], lw[2], lw[3]);
+                }
+            }
+        }
+        fence_async_smem();
+        mbar_arrive(bar_u);
+        // gamma + b2 -> top-k
+        mbar_wait(bar_g, 0, status, &abort_flag, 27);
+        tc_fence_after();
+        __syncwarp();
+        uint32_t sr[32];
+        tmem_ld32(lane_base + 320, sr);
+        tmem_wait_ld();
+        if (routed && !abort_flag) {
+            float gam[kG];
+#pragma unroll
+            for (int g = 0; g < kG; ++g) gam[g] = __uint_as_float(sr[g]) + __ldg(b2 + (int64_t)l * kG + g);
+            const int k = sg.k;
+            uint8_t *dst = idx + (int64_t)l * idx_per_layer + sg.idx_off + (r - sg.token_row) * k;
+            int pos = 0;
+#pragma unroll
+            for (int g = 0; g < kG; ++g) {
+                int rank = 0;
+#pragma unroll
+                for (int g2 = 0; g2 < kG; ++g2)
+                    rank += (gam[g2] > gam[g] || (gam[g2] == gam[g] && g2 < g)) ? 1 : 0;
+                if (rank < k) dst[pos++] = (uint8_t)g;
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, 512);
+    }
+}
+
+}  // namespace
+
+bool router_tc_supported(const rolesub_shape *s)
+{
+    const int d = s->num_heads * s->head_dim;
+    return s->dtype == ROLESUB_BF16 && s->router_hidden == kF && s->role_dim == kC && s->num_groups == kG &&
+           d % 64 == 0;
+}
+
+cudaError_t launch_router_tc(const CompressArgs &a)
+{
+    const rolesub_shape &S = *a.shape;
+    const rolesub_plan &P = *a.plan.hdr;
+    if (P.num_route_tiles == 0) return cudaSuccess;
+    const int L = S.num_layers, d = S.num_heads * S.head_dim;
+    const int64_t rows = P.rows_per_layer;
+    const int64_t w1cols = 2 * (int64_t)d + kC;
+    CUtensorMap th, tw1, twre, tw2;
+    {
+        const uint64_t dims[3] = {(uint64_t)d, (uint64_t)rows, (uint64_t)L};
+        const uint64_t str[2] = {(uint64_t)d * 2, (uint64_t)(rows * d * 2)};
+        const uint32_t box[3] = {64, (uint32_t)kRows, 1};
+        if (!make_bf16_map(&th, a.h, 3, dims, str, box)) return cudaErrorInvalidValue;
+    }
+    {
+        const uint64_t dims[3] = {(uint64_t)w1cols, (uint64_t)kF, (uint64_t)L};
+        const uint64_t str[2] = {(uint64_t)w1cols * 2, (uint64_t)(w1cols * kF * 2)};
+        const uint32_t box[3] = {64, (uint32_t)kF, 1};
+        if (!make_bf16_map(&tw1, a.W1, 3, dims, str, box)) return cudaErrorInvalidValue;
+    }
+    {
+        const uint64_t dims[3] = {(uint64_t)d, (uint64_t)kC, (uint64_t)L};
+        const uint64_t str[2] = {(uint64_t)d * 2, (uint64_t)d * kC * 2};
+        const uint32_t box[3] = {64, (uint32_t)kC, 1};
+        if (!make_bf16_map(&twre, a.W_re, 3, dims, str, box)) return cudaErrorInvalidValue;
+    }
+    {
+        const uint64_t dims[3] = {(uint64_t)kF, (uint64_t)kG, (uint64_t)L};
+        const uint64_t str[2] = {(uint64_t)kF * 2, (uint64_t)kF * kG * 2};
+        const uint32_t box[3] = {64, (uint32_t)kG, 1};
+        if (!make_bf16_map(&tw2, a.W2, 3, dims, str, box)) return cudaErrorInvalidValue;
+    }
+    cudaError_t err = cudaFuncSetAttribute(k_router_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (err != cudaSuccess) return err;
+    PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev,
+               a.plan.route_tiles_dev};
+    k_router_tc<<<dim3((unsigned)P.num_route_tiles, L), kThreads, kSmemBytes, a.stream>>>(
+        th, tw1, twre, tw2, pd, rows, d, P.num_episodes, S.num_groups, a.b_re, a.ws.lang_bias, a.b2, a.alpha_role,
+        a.idx, P.idx_bytes_per_layer, a.ws.status);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+}  // namespace rs

@@ -73,7 +73,9 @@ class PlanHeader(ctypes.Structure):
                 ("num_groups", ctypes.c_int32), ("reserved", ctypes.c_int32),
                 ("off_segments", ctypes.c_int64), ("off_episodes", ctypes.c_int64),
                 ("off_row_seg", ctypes.c_int64), ("off_routed_rows", ctypes.c_int64),
-                ("off_stored_rows", ctypes.c_int64), ("total_bytes", ctypes.c_int64)]
+                ("off_stored_rows", ctypes.c_int64), ("total_bytes", ctypes.c_int64),
+                ("num_route_tiles", ctypes.c_int32), ("reserved2", ctypes.c_int32),
+                ("off_route_tiles", ctypes.c_int64)]
 
 
 _vp = ctypes.c_void_p

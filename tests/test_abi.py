@@ -45,7 +45,7 @@ def test_struct_sizes_match_header(rsm):
     assert ctypes.sizeof(rsm.Shape) == 32
     assert ctypes.sizeof(rsm.Segment) == 40
     assert ctypes.sizeof(rsm.Episode) == 40
-    assert ctypes.sizeof(rsm.PlanHeader) == 136
+    assert ctypes.sizeof(rsm.PlanHeader) == 152
 
 
 def _plan(rsm, n_tok, k, n_q, H=2, dh=8, G=4, dtype="f32"):
@@ -87,6 +87,15 @@ def test_plan_matches_oracle_layout(rsm, oracle):
         assert all(0 < kk[rs_[r]] < G for r in rr) and all(kk[rs_[r]] > 0 for r in sr)
         for s, seg in enumerate(p.segments):
             assert np.all(rs_[seg.token_row:seg.token_row + seg.n_tokens] == s)
+        # router tiles: 128-row windows that start on routed rows and cover
+        # every routed row exactly once
+        nt = h.num_route_tiles
+        tiles = np.frombuffer(p.host[h.off_route_tiles:h.off_route_tiles + 4 * nt].tobytes(), np.int32)
+        assert np.all(np.isin(tiles, rr)) and np.all(np.diff(tiles) >= 128)
+        cover = np.zeros(h.rows_per_layer, int)
+        for t0 in tiles:
+            cover[t0:t0 + 128] += 1
+        assert np.all(cover[rr] == 1)
 
 
 def test_plan_reproduces_table_1_visual_kv(rsm):
