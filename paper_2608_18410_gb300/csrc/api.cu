@@ -87,7 +87,7 @@ rolesub_status view_plan(const rolesub_shape *s, const void *plan_host, const vo
 }
 
 struct WsSizes {
-    size_t status, ctx, bias, logits, total;
+    size_t status, ctx, bias, logits, rowst, total;
 };
 
 WsSizes ws_sizes(const rolesub_shape *s, const rolesub_plan *p)
@@ -105,7 +105,8 @@ WsSizes ws_sizes(const rolesub_shape *s, const rolesub_plan *p)
                    : align_up(sizeof(float) * L * (size_t)p->routed_rows_per_layer *
                                   (size_t)(s->router_hidden + s->role_dim),
                               kAlign);
-    w.total = w.status + w.ctx + w.bias + w.logits;
+    w.rowst = rs::rotate_tc_supported(s) ? align_up((size_t)16 * L * (size_t)p->rows_per_layer, kAlign) : 0;
+    w.total = w.status + w.ctx + w.bias + w.logits + w.rowst;
     return w;
 }
 
@@ -117,6 +118,7 @@ Workspace carve(const WsSizes &w, void *base)
     ws.lang_ctx = (float *)(b + w.status);
     ws.lang_bias = (float *)(b + w.status + w.ctx);
     ws.logits = (float *)(b + w.status + w.ctx + w.bias);
+    ws.row_store = b + w.status + w.ctx + w.bias + w.logits;
     ws.bytes = w.total;
     return ws;
 }

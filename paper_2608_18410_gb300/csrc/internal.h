@@ -29,6 +29,7 @@ struct Workspace {  // carve-up of the caller's workspace
     float *lang_ctx;   // [L][E][d]
     float *lang_bias;  // [L][E][F]
     float *logits;     // [L][routed][F + C]   (router GEMM output)
+    void *row_store;   // [L][rows] 16-byte store records (tensor-core rotation)
     size_t bytes;
 };
 

@@ -1,18 +1,22 @@
 // rotate_tc.cu -- orthogonal value decomposition and packing (Sec. 3.2) on
 // the 5th-generation tensor core, bf16 inputs, fp32 accumulation.
 //
-// z = R_h^T v for every cache row and head, in row form Z_h = V_h R_h:
+// z = R_h^T v for every cache row and head, in row form Z = V_h R_h:
 //   A = 128 value rows of head h (K-major, TMA from v),
 //   B = R_h with B[n][k] = R_h[k][n]: R_h is row-major in k, so it is the
-//       MN-major operand, loaded by TMA as two 64-column blocks,
-//   D = 128 x 128 fp32 in TMEM (double buffered across heads).
+//       MN-major operand (two 64-column blocks loaded by TMA),
+//   D = 128 x 128 fp32 in TMEM.
 // The epilogue (one row per thread) keeps only the row's kept groups: each
 // group of d_s = 8 values becomes one 16-byte bf16 store into
 // packed[seg][h][i][j][:]. Segments with k = S also get indices 0..S-1.
 //
-// Grid: (128-row tiles of the layer, head groups, layers); each CTA loops
-// over `hpb` heads with a two-stage TMA/MMA pipeline so that loading and
-// multiplying head h+1 overlaps the epilogue of head h.
+// One CTA per (head, layer, range of 128-row tiles), 192 threads:
+//   warp 4  TMA producer: R_h once, then value tiles into a 4-stage ring
+//   warp 5  MMA issuer: one 128x128x128 MMA per tile, TMEM double-buffered
+//   warps 0-3 epilogue: TMEM -> bf16 group stores; the next tile's row
+//           metadata (segment, kept groups) is fetched ahead of time
+// R_h stays in shared memory for the CTA's lifetime, so it is read from
+// L2 once per (head, layer, range) instead of once per tile.
 #include <cuda.h>
 
 #include "common.cuh"
@@ -26,71 +30,92 @@ namespace {
 using namespace sm100;
 typedef __nv_bfloat16 bf16;
 
-constexpr int kThreads = 128;
+constexpr int kThreads = 192;
 constexpr int kRows = 128;
 constexpr int kDh = 128;
 constexpr int kG = 16;
+constexpr int kStages = 4;
 
-constexpr uint32_t kStage = 65536;           // V tile (32K) + R_h (32K)
-constexpr uint32_t kOffBar = 2 * kStage;
-constexpr uint32_t kSmemBytes = kOffBar + 128 + 1024;
+constexpr uint32_t kOffR = 0;                       // R_h: 2 x 16K (MN-blocks)
+constexpr uint32_t kOffV = 32768;                   // V ring: 4 x 32K
+constexpr uint32_t kVBytes = 32768;
+constexpr uint32_t kOffZ = kOffV + kStages * kVBytes;   // bf16 z rows: 128 x 256 B
+constexpr uint32_t kOffBar = kOffZ + 32768;
+constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kIdesc = idesc_bf16(128, 128, true);
 
-__device__ __forceinline__ void store_group(bf16 *dst, const uint32_t (&sr)[32], int w)
+// Per-row store record, built once per (layer, row) by k_row_store:
+//   x, y: kept group ids, 4 bits each in storage order (64 bits)
+//   z:    (packed_off + i * k * d_s) / 8, the row's first group for head 0
+//   w:    k << 27 | n * k, i.e. kept groups and the per-head stride / 8
+// k = 0 means nothing is stored for the row (or its indices were corrupt).
+__global__ void __launch_bounds__(256)
+k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_per_layer,
+            uint4 *__restrict__ meta, int32_t *status)
 {
-    // columns 8w .. 8w+7 of this 32-column slice
-    uint32_t a, b, c, d;
-#define RS_PACK(o)                                                                   \
-    a = pack_bf16(__uint_as_float(sr[o + 0]), __uint_as_float(sr[o + 1]));           \
-    b = pack_bf16(__uint_as_float(sr[o + 2]), __uint_as_float(sr[o + 3]));           \
-    c = pack_bf16(__uint_as_float(sr[o + 4]), __uint_as_float(sr[o + 5]));           \
-    d = pack_bf16(__uint_as_float(sr[o + 6]), __uint_as_float(sr[o + 7]));
-    switch (w) {
-    case 0: RS_PACK(0); break;
-    case 1: RS_PACK(8); break;
-    case 2: RS_PACK(16); break;
-    default: RS_PACK(24); break;
+    const int l = blockIdx.y;
+    const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (r >= rows) return;
+    const rolesub_segment sg = plan.segs[plan.row_seg[r]];
+    const int k = sg.k;
+    const int64_t ti = r - sg.token_row;
+    uint8_t *ix = idx + (int64_t)l * idx_per_layer + sg.idx_off + ti * k;
+    uint64_t gid = 0;
+    int kk = k;
+    if (k == kG) {
+        gid = 0xFEDCBA9876543210ull;
+        for (int s = 0; s < kG; ++s) ix[s] = (uint8_t)s;   // byte stores: no alignment needed
+    } else {
+        for (int s = 0; s < k; ++s) {
+            const uint32_t g = ix[s];
+            if (g >= kG) {
+                report(status, ROLESUB_EDEVICE, (int)r);
+                kk = 0;
+                break;
+            }
+            gid |= (uint64_t)g << (4 * s);
+        }
     }
-#undef RS_PACK
-    *reinterpret_cast<uint4 *>(dst) = make_uint4(a, b, c, d);
+    const int64_t base8 = sg.packed_off / 8 + ti * k;
+    meta[(int64_t)l * rows + r] = make_uint4((uint32_t)gid, (uint32_t)(gid >> 32), (uint32_t)base8,
+                                             ((uint32_t)kk << 27) | (uint32_t)((int64_t)sg.n_tokens * k));
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_r, PlanDev plan,
-            int64_t rows, int H, int hpb, bf16 *__restrict__ packed, int64_t packed_per_layer,
-            uint8_t *__restrict__ idx, int64_t idx_per_layer, int32_t *status)
+k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_r,
+            const uint4 *__restrict__ meta, int64_t rows, int H, int tiles_per_cta, int ntiles,
+            bf16 *__restrict__ packed, int64_t packed_per_layer, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint32_t tmem_slot;
     __shared__ volatile int abort_flag;
     const uint32_t sraw = smem_u32(smem_raw);
     const uint32_t sb = (sraw + 1023u) & ~1023u;
-    const int tid = threadIdx.x, warp = tid >> 5;
-    const int l = blockIdx.z;
-    const int64_t r0 = (int64_t)blockIdx.x * kRows;
-    const int h0 = blockIdx.y * hpb;
-    const int nh = min(hpb, H - h0);
-    if (nh <= 0) return;
-    const uint32_t bar_full = sb + kOffBar, bar_done = bar_full + 16;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int h = blockIdx.x, l = blockIdx.y;
+    const int t0 = blockIdx.z * tiles_per_cta;
+    const int nt = min(tiles_per_cta, ntiles - t0);
+    if (nt <= 0) return;
 
-    auto load_head = [&](int i) {  // stage i & 1 <- V tile and R of head h0 + i
-        const uint32_t st = sb + kStage * (uint32_t)(i & 1);
-        const int h = h0 + i;
-        mbar_expect_tx(bar_full + 8 * (i & 1), 65536);
-        tma_load_4d(st, &tm_v, 0, h, (int)r0, l, bar_full + 8 * (i & 1));
-        tma_load_4d(st + 16384, &tm_v, 64, h, (int)r0, l, bar_full + 8 * (i & 1));
-        tma_load_3d(st + 32768, &tm_r, 0, 0, l * H + h, bar_full + 8 * (i & 1));
-        tma_load_3d(st + 49152, &tm_r, 64, 0, l * H + h, bar_full + 8 * (i & 1));
-    };
+    const uint32_t bar_r = sb + kOffBar;
+    const uint32_t bar_full = bar_r + 8;                 // [4]
+    const uint32_t bar_empty = bar_full + 32;            // [4]
+    const uint32_t bar_tfull = bar_empty + 32;           // [2]
+    const uint32_t bar_tempty = bar_tfull + 16;          // [2]
+
     if (tid == 0) {
         abort_flag = 0;
-        for (int i = 0; i < 4; ++i) mbar_init(bar_full + 8 * i, 1);
+        mbar_init(bar_r, 1);
+        for (int i = 0; i < kStages; ++i) {
+            mbar_init(bar_full + 8 * i, 1);
+            mbar_init(bar_empty + 8 * i, 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar_tfull + 8 * i, 1);
+            mbar_init(bar_tempty + 8 * i, 128);
+        }
         fence_mbar_init();
-        prefetch_tmap(&tm_v);
-        prefetch_tmap(&tm_r);
-        load_head(0);
-        if (nh > 1) load_head(1);
     }
     __syncthreads();
     if (warp == 0) {
@@ -102,71 +127,100 @@ k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CU
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
-    auto issue_mma = [&](int i) {
-        const uint32_t st = sb + kStage * (uint32_t)(i & 1);
-        if (!mbar_wait(bar_full + 8 * (i & 1), (i >> 1) & 1, status, &abort_flag, 10)) return;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-            const uint64_t a = sdesc_sw128(st + (kk >> 2) * 16384u + (kk & 3) * 32u, 16, 1024);
-            const uint64_t b = sdesc_sw128(st + 32768u + 2048u * kk, 16384, 1024);
-            mma_bf16(tmem + 128u * (i & 1), a, b, kIdesc, kk > 0);
+    if (warp == 4) {
+        if (lane == 0) {
+            prefetch_tmap(&tm_v);
+            prefetch_tmap(&tm_r);
+            mbar_expect_tx(bar_r, 32768);
+            tma_load_3d(sb + kOffR, &tm_r, 0, 0, l * H + h, bar_r);
+            tma_load_3d(sb + kOffR + 16384, &tm_r, 64, 0, l * H + h, bar_r);
+            for (int t = 0; t < nt; ++t) {
+                const int s = t % kStages;
+                if (t >= kStages && !mbar_wait(bar_empty + 8 * s, ((t / kStages) - 1) & 1, status, &abort_flag, 30))
+                    break;
+                const uint32_t st = sb + kOffV + kVBytes * s;
+                const int r0 = (t0 + t) * kRows;
+                mbar_expect_tx(bar_full + 8 * s, kVBytes);
+                tma_load_4d(st, &tm_v, 0, h, r0, l, bar_full + 8 * s);
+                tma_load_4d(st + 16384, &tm_v, 64, h, r0, l, bar_full + 8 * s);
+            }
         }
-        mma_commit(bar_done + 8 * (i & 1));
-    };
-    if (tid == 0) issue_mma(0);
-
-    // this thread's row: segment, kept groups
-    const int64_t r = r0 + tid;
-    int k = 0;
-    rolesub_segment sg{};
-    int gid[kG];
-    if (r < rows) {
-        sg = plan.segs[plan.row_seg[r]];
-        k = sg.k;
-    }
-    const int64_t ti = r - sg.token_row;
-    uint8_t *ix = idx + (int64_t)l * idx_per_layer + sg.idx_off + ti * k;
+    } else if (warp == 5) {
+        if (lane == 0 && mbar_wait(bar_r, 0, status, &abort_flag, 31)) {
+            for (int t = 0; t < nt; ++t) {
+                const int s = t % kStages, b = t & 1;
+                if (!mbar_wait(bar_full + 8 * s, (t / kStages) & 1, status, &abort_flag, 32)) break;
+                if (t >= 2 && !mbar_wait(bar_tempty + 8 * b, ((t >> 1) - 1) & 1, status, &abort_flag, 33)) break;
+                tc_fence_after();
+                const uint32_t st = sb + kOffV + kVBytes * s;
 #pragma unroll
-    for (int s = 0; s < kG; ++s) gid[s] = s;
-    if (k > 0 && k < kG) {
-#pragma unroll
-        for (int s = 0; s < kG; ++s)
-            if (s < k) gid[s] = ix[s];
-    }
-    if (k == kG && blockIdx.y == 0) {   // byte stores: idx offsets need no alignment
-#pragma unroll
-        for (int s = 0; s < kG; ++s) ix[s] = (uint8_t)s;
-    }
-    bool bad = false;
-#pragma unroll
-    for (int s = 0; s < kG; ++s)
-        if (s < k && gid[s] >= kG) bad = true;
-    if (bad) report(status, ROLESUB_EDEVICE, (int)r);
-
-    for (int i = 0; i < nh; ++i) {
-        const int h = h0 + i;
-        if (tid == 0 && !abort_flag && i + 1 < nh) issue_mma(i + 1);  // overlaps this head's epilogue
-        mbar_wait(bar_done + 8 * (i & 1), (i >> 1) & 1, status, &abort_flag, 11);
-        tc_fence_after();
-        if (tid == 0 && !abort_flag && i + 2 < nh) load_head(i + 2);   // stage i & 1 is free
-        __syncwarp();
-        bf16 *dst = packed + (int64_t)l * packed_per_layer + sg.packed_off + ((int64_t)h * sg.n_tokens + ti) * k * 8;
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-            uint32_t sr[32];
-            tmem_ld32(tmem + ((uint32_t)(32 * warp) << 16) + 128u * (i & 1) + 32u * q4, sr);
-            tmem_wait_ld();
-            if (bad || abort_flag) continue;
-#pragma unroll
-            for (int s = 0; s < kG; ++s)
-                if (s < k && (gid[s] >> 2) == q4) store_group(dst + 8 * s, sr, gid[s] & 3);
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint64_t a = sdesc_sw128(st + (kk >> 2) * 16384u + (kk & 3) * 32u, 16, 1024);
+                    const uint64_t bd = sdesc_sw128(sb + kOffR + 2048u * kk, 16384, 1024);
+                    mma_bf16(tmem + 128u * b, a, bd, kIdesc, kk > 0);
+                }
+                mma_commit(bar_empty + 8 * s);
+                mma_commit(bar_tfull + 8 * b);
+            }
         }
-        tc_fence_before();
-        __syncthreads();   // TMEM buffer i & 1 may be overwritten by head i + 2
-        tc_fence_after();
+    } else {
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
+        // row records of this thread's row in tiles t, t+1 (t+2 is fetched
+        // during tile t, so the load latency hides behind two tiles of work)
+        const uint4 *mrow = meta + (int64_t)l * rows + (int64_t)t0 * kRows + tid;
+        const uint4 zero4 = make_uint4(0, 0, 0, 0);
+        const int64_t rfirst = (int64_t)t0 * kRows + tid;
+        uint4 m0 = rfirst < rows ? __ldg(mrow) : zero4;
+        uint4 m1 = (nt > 1 && rfirst + kRows < rows) ? __ldg(mrow + kRows) : zero4;
+        bf16 *pl = packed + (int64_t)l * packed_per_layer;
+        for (int t = 0; t < nt; ++t) {
+            const int b = t & 1;
+            const int64_t r2 = rfirst + (int64_t)(t + 2) * kRows;
+            const uint4 m2 = (t + 2 < nt && r2 < rows) ? __ldg(mrow + (int64_t)(t + 2) * kRows) : zero4;
+            mbar_wait(bar_tfull + 8 * b, (t >> 1) & 1, status, &abort_flag, 34);
+            tc_fence_after();
+            __syncwarp();
+            const uint64_t gid = (uint64_t)m0.x | ((uint64_t)m0.y << 32);
+            const int k = abort_flag ? 0 : (int)(m0.w >> 27);
+            uint4 *dst = reinterpret_cast<uint4 *>(pl + ((int64_t)m0.z + (int64_t)h * (int64_t)(m0.w & 0x7FFFFFFu)) * 8);
+            // the row's z as 16 bf16 chunks (one per group) in shared memory,
+            // chunk c at position c ^ (row & 15) to spread banks
+            const uint32_t zrow = sb + kOffZ + (uint32_t)tid * 256u;
+            const uint32_t sw = (uint32_t)(tid & 15);
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                uint32_t sa[32], sc[32];
+                tmem_ld32(lane_base + 128u * b + 64u * half, sa);
+                tmem_ld32(lane_base + 128u * b + 64u * half + 32u, sc);
+                tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < 8; ++c) {
+                    const uint32_t(&src)[32] = c < 4 ? sa : sc;
+                    const int o = 8 * (c & 3);
+                    st_shared_v4(zrow + ((((uint32_t)(8 * half + c)) ^ sw) << 4),
+                                 pack_bf16(__uint_as_float(src[o]), __uint_as_float(src[o + 1])),
+                                 pack_bf16(__uint_as_float(src[o + 2]), __uint_as_float(src[o + 3])),
+                                 pack_bf16(__uint_as_float(src[o + 4]), __uint_as_float(src[o + 5])),
+                                 pack_bf16(__uint_as_float(src[o + 6]), __uint_as_float(src[o + 7])));
+                }
+            }
+            tc_fence_before();
+            mbar_arrive(bar_tempty + 8 * b);   // TMEM buffer b is free for tile t + 2
+            // kept groups in storage order: same-thread shared-memory round trip
+            for (int s = 0; s < k; ++s) {
+                const uint32_t g = (uint32_t)(gid >> (4 * s)) & 15u;
+                dst[s] = ld_shared_v4(zrow + ((g ^ sw) << 4));
+            }
+            m0 = m1;
+            m1 = m2;
+        }
     }
-    if (warp == 0) tmem_dealloc(tmem, kTmemCols);
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) {
+        tc_fence_after();
+        tmem_dealloc(tmem, kTmemCols);
+    }
 }
 
 }  // namespace
@@ -198,16 +252,20 @@ cudaError_t launch_rotate_tc(const CompressArgs &a)
     }
     cudaError_t err = cudaFuncSetAttribute(k_rotate_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (err != cudaSuccess) return err;
-    const int64_t tiles = (rows + kRows - 1) / kRows;
-    // heads per CTA: enough CTAs to fill the GPU twice over, otherwise all heads
-    int hpb = H;
-    const int64_t units = tiles * L;
-    while (hpb > 1 && units * ((H + hpb - 1) / hpb) < 2 * 152) hpb = (hpb + 1) / 2;
-    PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev};
-    k_rotate_tc<<<dim3((unsigned)tiles, (H + hpb - 1) / hpb, L), kThreads, kSmemBytes, a.stream>>>(
-        tv, tr, pd, rows, H, hpb, (bf16 *)a.packed, P.packed_elems_per_layer, a.idx, P.idx_bytes_per_layer,
-        a.ws.status);
-    count_launches(1);
+    const int ntiles = (int)((rows + kRows - 1) / kRows);
+    // split each (head, layer) tile list so that there are at least ~4 CTAs per SM-wave
+    int splits = 1;
+    while ((int64_t)H * L * splits < 4 * 152 && splits < ntiles) ++splits;
+    const int per = (ntiles + splits - 1) / splits;
+    splits = (ntiles + per - 1) / per;
+    PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev,
+               a.plan.route_tiles_dev};
+    uint4 *meta = reinterpret_cast<uint4 *>(a.ws.row_store);
+    k_row_store<<<dim3((unsigned)((rows + 255) / 256), L), 256, 0, a.stream>>>(pd, rows, a.idx,
+                                                                              P.idx_bytes_per_layer, meta, a.ws.status);
+    k_rotate_tc<<<dim3(H, L, splits), kThreads, kSmemBytes, a.stream>>>(
+        tv, tr, meta, rows, H, per, ntiles, (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
+    count_launches(2);
     return cudaGetLastError();
 }
 

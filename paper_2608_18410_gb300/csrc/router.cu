@@ -31,22 +31,53 @@ __global__ void k_lang_pool(const T *__restrict__ h, const rolesub_episode *__re
 }
 
 // beta[l][e][f] = b1[f] + alpha_lang * W1[f][d+C : 2d+C] . ctx[l][e]
+// A small GEMM per layer (episodes x F x d): 16 episodes x 64 outputs per
+// block, the hidden dimension streamed through shared memory in 64-wide
+// steps; every thread owns one episode and four outputs.
 template <class T>
-__global__ void k_lang_bias(const T *__restrict__ W1, const float *__restrict__ b1,
-                            const float *__restrict__ ctx, int E, int d, int C, int F,
-                            float alpha_lang, float *__restrict__ beta)
+__global__ void __launch_bounds__(256)
+k_lang_bias(const T *__restrict__ W1, const float *__restrict__ b1, const float *__restrict__ ctx,
+            int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
 {
-    const int l = blockIdx.y;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int f = blockIdx.x * (blockDim.x >> 5) + warp;
-    if (f >= F) return;
-    const T *w = W1 + ((size_t)l * F + f) * (size_t)(2 * d + C) + d + C;
-    for (int e = 0; e < E; ++e) {
-        const float *ce = ctx + ((size_t)l * E + e) * d;
-        float s = 0.f;
-        for (int t = lane; t < d; t += 32) s += to_f(w[t]) * ce[t];
-        s = warp_sum(s);
-        if (lane == 0) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * s;
+    constexpr int BE = 16, BF = 64, BK = 64, WP = BF + 4;   // WP: padded row pitch
+    __shared__ __align__(16) float Ws[BK * WP];             // [t][f]
+    __shared__ float Cs[BE][BK + 1];                        // [e][t]
+    const int l = blockIdx.z;
+    const int f0 = blockIdx.x * BF, e0 = blockIdx.y * BE;
+    const int te = threadIdx.x >> 4, tf = threadIdx.x & 15;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    const size_t wstride = (size_t)(2 * d + C);
+    for (int k0 = 0; k0 < d; k0 += BK) {
+        for (int i = threadIdx.x; i < BF * BK; i += 256) {
+            const int ff = i / BK, t = i % BK;
+            const int f = f0 + ff;
+            Ws[t * WP + ff] = (f < F && k0 + t < d)
+                                   ? to_f(W1[((size_t)l * F + f) * wstride + d + C + k0 + t])
+                                   : 0.f;
+        }
+        for (int i = threadIdx.x; i < BE * BK; i += 256) {
+            const int ee = i / BK, t = i % BK;
+            const int e = e0 + ee;
+            Cs[ee][t] = (e < E && k0 + t < d) ? ctx[((size_t)l * E + e) * d + k0 + t] : 0.f;
+        }
+        __syncthreads();
+#pragma unroll 16
+        for (int t = 0; t < BK; ++t) {
+            const float c = Cs[te][t];
+            const float4 w = *reinterpret_cast<const float4 *>(&Ws[t * WP + 4 * tf]);
+            acc[0] = fmaf(c, w.x, acc[0]);
+            acc[1] = fmaf(c, w.y, acc[1]);
+            acc[2] = fmaf(c, w.z, acc[2]);
+            acc[3] = fmaf(c, w.w, acc[3]);
+        }
+        __syncthreads();
+    }
+    const int e = e0 + te;
+    if (e >= E) return;
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+        const int f = f0 + 4 * tf + j;
+        if (f < F) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * acc[j];
     }
 }
 
@@ -200,7 +231,7 @@ static cudaError_t launch_router_t(const CompressArgs &a)
             *W2 = (const T *)a.W2;
     k_lang_pool<T><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
         h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
-    k_lang_bias<T><<<dim3((F + 7) / 8, L), 256, 0, a.stream>>>(
+    k_lang_bias<T><<<dim3((F + 63) / 64, (E + 15) / 16, L), 256, 0, a.stream>>>(
         W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
     if (router_tc_supported(a.shape)) {
         count_launches(2);
