@@ -210,6 +210,14 @@ def max_over_ranks(x, ws):
     return float(t.item())
 
 
+def weak_scaling(total_ms_local, steps, query_tokens_per_step, ws):
+    """Whole-job throughput over ranks that each process their own batch:
+    the slowest rank's time bounds the job; every rank's tokens count."""
+    total_ms = max_over_ranks(total_ms_local, ws)
+    ms_per_step = total_ms / steps
+    return ms_per_step, query_tokens_per_step * ws / (ms_per_step / 1e3)
+
+
 def barrier(ws):
     if ws > 1:
         import torch.distributed as dist
@@ -370,10 +378,8 @@ def run_ours(args):
     t_comp = [a.elapsed_time(b) for a, b, c in ev]
     t_att = [b.elapsed_time(c) for a, b, c in ev]
     t_step = [x + y for x, y in zip(t_comp, t_att)]
-    total_ms = max_over_ranks(sum(t_step), ws)
-    ms_per_step = total_ms / args.steps
     qtok = wl.q_rows * wl.L
-    value = qtok * ws / (ms_per_step / 1e3)
+    ms_per_step, value = weak_scaling(sum(t_step), args.steps, qtok, ws)
 
     # ---- end to end through the public API from pinned host buffers --------
     act = ("h", "v", "K", "q")
