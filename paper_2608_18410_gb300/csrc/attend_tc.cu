@@ -1,30 +1,64 @@
 // attend_tc.cu -- attention over the routed value cache on the 5th-generation
 // tensor core (tcgen05 + TMA), bf16 inputs, fp32 accumulation.
 //
-// One CTA per (layer, episode, head, tile of 64 queries); 128 threads.
-// Per chunk c of 64 cache tokens:
-//   S_c = Q K_c^T                 tcgen05 MMA, M=128 (rows >= 64 unused),
-//                                 N=64, K=128; K_c staged by TMA (double
-//                                 buffered) straight from the caller's cache
-//   online softmax (warps 0-1, one query row per thread, exp2 domain):
-//     m_c = max(m_{c-1}, rowmax S_c), P_c = exp(S_c - m_c) (bf16, smem)
-//   Z_c = the chunk's packed kept groups scattered by their indices into a
-//         zero-filled 64 x 128 tile (warps 2-3; MN-major, 16-byte stores:
-//         one group of d_s = 8 bf16 is exactly one swizzle chunk)
-//   Y_c = P_c Z_c                  tcgen05 MMA into TMEM; accumulated into
-//                                 registers as y = y * exp(m_{c-1} - m_c) + Y_c
-// Finally y /= l, O = Y R_h^T on the tensor core (o_q = R_h y_q, Sec. 3.2),
-// and each thread stores its 256-byte output row.
+// Work unit = (layer, head, episode, tile of 64 queries). A persistent CTA
+// per SM walks a contiguous range of units (episode fastest), so R_h stays
+// in shared memory while (layer, head) is unchanged.
 //
-// Shared memory (1024-aligned, 72 KB, two CTAs per SM):
-//   [0,16K)    Q (two 64-column K-blocks at +0, +8K), later Y (bf16)
-//   [16K,48K)  K chunk buffers 2 x 16K; after the last S MMA, R_h (32K)
-//   [48K,56K)  P chunk (64 rows x 64 kv)
-//   [56K,72K)  Z chunk (two 64-column MN-blocks of 64 kv rows)
-// M=128 MMAs read 128 A rows; rows 64..127 of Q/Y/P fall on the next
-// region and only produce output rows that are never read.
-// TMEM (256 columns): S buffers at 0 and 64, Y_c at 128, O at 0.
+// All products are M = 64 (the 64 query rows of a unit): their TMEM
+// accumulators put rows 16q..16q+15 in lanes 32q..32q+15, so each of the
+// four lane quadrants -- one per SM sub-partition -- holds 16 complete rows
+// and one warp per quadrant does that quadrant's softmax with row maxima
+// reduced by shuffles inside the warp (16x256b TMEM loads: thread t holds
+// rows t/4 and t/4 + 8, column pairs 8j + 2(t%4)).
+//
+// Per chunk c of 64 cache tokens of a unit:
+//   S_c = Q K_c^T                 tcgen05, M=64, N=64, K=128; K_c by TMA
+//                                 straight from the caller's cache
+//   softmax, exp2 domain:         P_c = exp(S_c - m) -> bf16 smem, with a
+//                                 reference max m per row that is raised
+//                                 (and the TMEM accumulator Y rescaled) only
+//                                 when a chunk's row max exceeds it by more
+//                                 than 2^8; Y and the row sum l always share
+//                                 the same m, so y / l is exact
+//   Z_c = the chunk's kept groups scattered by index into a zero-filled
+//         64 x 128 MN-major tile. One group of d_s = 8 bf16 is one 16-byte
+//         swizzle chunk, copied by cp.async from the packed cache straight
+//         to its slot; per-row records (kept ids, packed offset) are fetched
+//         three chunks ahead.
+//   Y += P_c Z_c                   tcgen05, M=64, N=128 (rotated space)
+// Unit tail: Y / l -> bf16 smem (into the unit's finished Q slot),
+// O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into the unit's Y buffer, output
+// stores.
+//
+// Warp roles (384 threads), all hand-offs through mbarriers:
+//   warps 0-3   softmax, one per TMEM lane quadrant
+//   warps 4,5   value gather, one kv row per thread
+//   warp 6      TMA producer: K (4-slot ring), Q (2 slots), R_h
+//   warp 7      MMA issuer: a non-blocking loop over three cursors (next S,
+//               next P.Z, next output product) that issues whichever is
+//               ready, in order within each cursor
+//   warps 8-11  unit tail, one per lane quadrant, overlapping the next
+//               unit's chunks (Y is double buffered in TMEM)
+// P is double buffered and Z has four slots: a chunk's softmax waits for the
+// product two chunks back, its gather for the one four chunks back, and the
+// gather publishes a chunk two iterations after issuing its copies.
+//
+// Shared memory (1024-aligned):
+//   0K   Q[2]   16K each (two 64-column K-blocks of 64 rows); the unit tail
+//                writes Y / l into its own Q slot
+//   32K  K[4]   16K each (64-row chunks)
+//   96K  R_h    32K (two 64-column K-blocks of 128 rows)
+//   128K P[2]   8K each (64 rows x 64 kv)
+//   144K Z[4]   16K each (two 64-column MN-blocks of 64 kv rows)
+//   208K records 4 x 1K
+//   212K row sums 2 x 64 fp32 (softmax -> unit tail)
+//   then the episode table and the barriers
+// TMEM (384 of 512 columns): S[2] at 0 and 64, Y[2] at 128 and 256 (each
+// later holding its unit's O).
 #include <cuda.h>
+
+#include <algorithm>
 
 #include "common.cuh"
 #include "internal.h"
@@ -37,94 +71,199 @@ namespace {
 using namespace sm100;
 typedef __nv_bfloat16 bf16;
 
-constexpr int kThreads = 128;
+constexpr int kThreads = 384;
 constexpr int kChunk = 64;   // cache tokens per chunk
-constexpr int kQRows = 64;   // query rows per CTA
+constexpr int kQRows = 64;   // query rows per unit
 constexpr int kDh = 128;
-constexpr int kG = 16;       // groups per head (d_s = 8: one 16-byte chunk)
+constexpr int kG = 16;       // groups per head (d_s = 8)
+constexpr int kMaxEp = 256;  // episodes per launch (episode table in smem)
+constexpr int kKSlots = 4;
+constexpr float kRescaleLog2 = 8.f;   // raise the reference max beyond 2^8 growth
 
 constexpr uint32_t kOffQ = 0;
-constexpr uint32_t kOffK = 16384;
-constexpr uint32_t kOffP = 49152;
-constexpr uint32_t kOffZ = 57344;
-constexpr uint32_t kOffBar = 73728;
-constexpr uint32_t kSmemBytes = kOffBar + 128 + 1024;  // + alignment slack
-constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kOffK = 32768;
+constexpr uint32_t kOffR = 98304;
+constexpr uint32_t kOffP = 131072;
+constexpr uint32_t kOffZ = 147456;                   // 4 x 16K ring
+constexpr int kZSlots = 4;
+constexpr uint32_t kOffRec = kOffZ + kZSlots * 16384; // 4 x 64 x 16 B
+constexpr uint32_t kOffL = kOffRec + 4096;           // 2 x 64 fp32 row sums
+constexpr uint32_t kOffEp = kOffL + 1024;            // 4 x kMaxEp int32
+constexpr uint32_t kOffBar = kOffEp + 16 * kMaxEp;
+constexpr uint32_t kSmemBytes = kOffBar + 512 + 1024;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColS = 0, kColY = 128;   // Y[b] at kColY + 128b
 
-constexpr uint32_t kIdescS = idesc_bf16(128, 64, false);
-constexpr uint32_t kIdescPV = idesc_bf16(128, 128, true);
-constexpr uint32_t kIdescO = idesc_bf16(128, 128, false);
+constexpr uint32_t kIdescS = idesc_bf16(64, 64, false);
+constexpr uint32_t kIdescPV = idesc_bf16(64, 128, true);
+constexpr uint32_t kIdescO = idesc_bf16(64, 128, false);
 
-__device__ __forceinline__ uint32_t tm_lane(uint32_t tmem, int warp, int col)
+// barrier slots (8 bytes each); [2] / [4] entries are per buffer
+enum {
+    B_QF = 0, B_QE = 2, B_KF = 4, B_KE = 8, B_RF = 12, B_RE = 13, B_SF = 14, B_PF = 16, B_ZF = 18, B_PV = 22,
+    B_YR = 26, B_YF = 28, B_OF = 29, B_OE = 30, B_LF = 32, B_COUNT = 34
+};
+
+struct Unit {
+    int l, h, e, nq, nc, nch, krow, qrow;
+};
+
+struct Ctx {
+    const int *ep_row, *ep_qrow, *ep_nc, *ep_nq;  // shared-memory episode table
+    int H, E, qtiles;
+};
+
+// Iterator over a CTA's units -- (layer, head, episode, query tile), query
+// tiles fastest, then episodes -- and over the chunks of each unit. Units
+// advance by counters (no division), so the iterator stays small wherever it
+// is inlined.
+struct ChunkIt {
+    int u, c, qt;   // unit index (u_end = done), chunk within unit, query tile
+    Unit t;
+};
+
+__device__ __forceinline__ void fill(const Ctx &x, ChunkIt &it)
 {
-    return tmem + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)col;
+    const int e = it.t.e, qb = it.qt * kQRows;
+    it.t.nq = max(0, min(kQRows, x.ep_nq[e] - qb));
+    it.t.nc = x.ep_nc[e];
+    it.t.nch = (it.t.nc + kChunk - 1) / kChunk;
+    it.t.krow = x.ep_row[e];
+    it.t.qrow = x.ep_qrow[e] + qb;
 }
 
-__global__ void __launch_bounds__(kThreads, 2)
+__device__ __forceinline__ void seek(const Ctx &x, ChunkIt &it, int u)
+{
+    it.u = u;
+    it.c = 0;
+    it.qt = u % x.qtiles;
+    int r = u / x.qtiles;
+    it.t.e = r % x.E;
+    r /= x.E;
+    it.t.h = r % x.H;
+    it.t.l = r / x.H;
+    fill(x, it);
+}
+
+__device__ __forceinline__ void step(const Ctx &x, ChunkIt &it)
+{
+    ++it.u;
+    if (++it.qt == x.qtiles) {
+        it.qt = 0;
+        if (++it.t.e == x.E) {
+            it.t.e = 0;
+            if (++it.t.h == x.H) {
+                it.t.h = 0;
+                ++it.t.l;
+            }
+        }
+    }
+    fill(x, it);
+}
+
+__device__ __forceinline__ bool busy(const Unit &t) { return t.nq > 0 && t.nc > 0; }
+
+__device__ __forceinline__ void skip_idle(const Ctx &x, ChunkIt &it, int u_end)
+{
+    while (it.u < u_end && !busy(it.t)) step(x, it);
+}
+
+__device__ __forceinline__ void it_first(const Ctx &x, ChunkIt &it, int u_begin, int u_end)
+{
+    seek(x, it, u_begin);
+    skip_idle(x, it, u_end);
+}
+
+// advances one chunk; returns true when it moved to another unit
+__device__ __forceinline__ bool it_next(const Ctx &x, ChunkIt &it, int u_end)
+{
+    if (it.u >= u_end) return false;
+    if (++it.c < it.t.nch) return false;
+    it.c = 0;
+    step(x, it);
+    skip_idle(x, it, u_end);
+    return true;
+}
+
+__device__ __forceinline__ void next_unit(const Ctx &x, ChunkIt &it, int u_end)
+{
+    it.c = it.t.nch - 1;
+    it_next(x, it, u_end);
+}
+
+__device__ __forceinline__ float quad_sum(float v)
+{
+    v += __shfl_xor_sync(0xffffffffu, v, 1);
+    return v + __shfl_xor_sync(0xffffffffu, v, 2);
+}
+
+__device__ __forceinline__ float quad_max(float v)
+{
+    v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 1));
+    return fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 2));
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
 k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
             const __grid_constant__ CUtensorMap tm_r, const bf16 *__restrict__ packed,
-            int64_t packed_per_layer, const uint8_t *__restrict__ idx, int64_t idx_per_layer,
-            PlanDev plan, int H, int qtiles, int64_t q_rows, float scale_log2,
-            bf16 *__restrict__ o, int32_t *status)
+            int64_t packed_per_layer, const uint4 *__restrict__ rec, int64_t rows,
+            const rolesub_episode *__restrict__ eps, int e0, int E, int H, int L, int qtiles, int64_t q_rows,
+            float scale_log2, bf16 *__restrict__ o, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ rolesub_segment sg[ROLESUB_NUM_KINDS];
-    __shared__ int row0[ROLESUB_NUM_KINDS + 1];
     __shared__ uint32_t tmem_slot;
     __shared__ volatile int abort_flag;
-
     const uint32_t sraw = smem_u32(smem_raw);
-    const uint32_t sb = (sraw + 1023u) & ~1023u;   // 1024-aligned base (swizzle atoms)
-    const int h = blockIdx.x, l = blockIdx.z;
-    const int e = blockIdx.y / qtiles, qt = blockIdx.y % qtiles;
-    const rolesub_episode ep = plan.eps[e];
-    const int qb = qt * kQRows;
-    if (qb >= ep.n_query) return;
-    const int nq = min(kQRows, ep.n_query - qb);
-    const int nc = ep.n_cache;
-    const int tid = threadIdx.x, warp = tid >> 5;
+    const uint32_t sb = (sraw + 1023u) & ~1023u;
+    uint8_t *sp = smem_raw + (sb - sraw);
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int64_t d = (int64_t)H * kDh;
 
-    if (nc == 0) {  // no cache tokens: o = 0
-        for (int i = tid; i < nq * (kDh / 8); i += kThreads) {
-            const int r = i / (kDh / 8), c8 = i % (kDh / 8);
-            uint4 *dst = reinterpret_cast<uint4 *>(o + ((int64_t)l * q_rows + ep.q_row_begin + qb + r) * d +
-                                                   (int64_t)h * kDh) + c8;
-            *dst = make_uint4(0, 0, 0, 0);
-        }
-        return;
+    // ---- episode table and unit range ------------------------------------
+    int *ep_tab = reinterpret_cast<int *>(sp + kOffEp);
+    for (int i = tid; i < E; i += kThreads) {
+        const rolesub_episode ep = eps[e0 + i];
+        ep_tab[i] = (int)ep.row_begin;
+        ep_tab[kMaxEp + i] = (int)ep.q_row_begin;
+        ep_tab[2 * kMaxEp + i] = ep.n_cache;
+        ep_tab[3 * kMaxEp + i] = ep.n_query;
     }
-    const int nchunks = (nc + kChunk - 1) / kChunk;
-    const uint32_t bar_q = sb + kOffBar, bar_k0 = bar_q + 8, bar_s0 = bar_q + 24, bar_pv = bar_q + 40,
-                   bar_r = bar_q + 48, bar_o = bar_q + 56;
-    const int krow0 = (int)ep.row_begin, qrow0 = (int)(ep.q_row_begin + qb);
+    const Ctx x{ep_tab, ep_tab + kMaxEp, ep_tab + 2 * kMaxEp, ep_tab + 3 * kMaxEp, H, E, qtiles};
+    const int64_t U = (int64_t)L * H * E * qtiles;
+    const int u_begin = (int)(U * blockIdx.x / gridDim.x);
+    const int u_end = (int)(U * (blockIdx.x + 1) / gridDim.x);
 
+    const uint32_t bar = sb + kOffBar;
+    auto B = [&](int i) { return bar + 8u * (uint32_t)i; };
     if (tid == 0) {
         abort_flag = 0;
-        for (int i = 0; i < 8; ++i) mbar_init(bar_q + 8 * i, 1);
+        for (int i = 0; i < B_COUNT; ++i) {
+            uint32_t cnt = 1;
+            if (i == B_PF || i == B_PF + 1 || i == B_YF || i == B_OE || i == B_OE + 1 || i == B_LF || i == B_LF + 1)
+                cnt = 128;
+            if (i >= B_ZF && i < B_ZF + kZSlots) cnt = 64;
+            mbar_init(B(i), cnt);
+        }
         fence_mbar_init();
-        prefetch_tmap(&tm_q);
-        prefetch_tmap(&tm_k);
-        prefetch_tmap(&tm_r);
-        mbar_expect_tx(bar_q, 16384);
-        tma_load_4d(sb + kOffQ, &tm_q, 0, h, qrow0, l, bar_q);
-        tma_load_4d(sb + kOffQ + 8192, &tm_q, 64, h, qrow0, l, bar_q);
-        for (int c = 0; c < 2 && c < nchunks; ++c) {
-            mbar_expect_tx(bar_k0 + 8 * c, 16384);
-            tma_load_4d(sb + kOffK + 16384 * c, &tm_k, 0, h, krow0 + kChunk * c, l, bar_k0 + 8 * c);
-            tma_load_4d(sb + kOffK + 16384 * c + 8192, &tm_k, 64, h, krow0 + kChunk * c, l, bar_k0 + 8 * c);
-        }
-    }
-    if (tid < ROLESUB_NUM_KINDS) sg[tid] = plan.segs[ep.seg_begin + tid];
-    if (tid == 0) {
-        int r = 0;
-        for (int m = 0; m < ROLESUB_NUM_KINDS; ++m) {
-            row0[m] = r;
-            r += plan.segs[ep.seg_begin + m].n_tokens;
-        }
-        row0[ROLESUB_NUM_KINDS] = r;
     }
     __syncthreads();
+
+    // units without cache tokens: o = 0
+    ChunkIt z;
+    seek(x, z, u_begin);
+    for (; z.u < u_end; step(x, z)) {
+        const Unit &t = z.t;
+        if (t.nq == 0 || t.nc > 0) continue;
+        for (int i = tid; i < t.nq * (kDh / 8); i += kThreads) {
+            const int r = i / (kDh / 8), c8 = i % (kDh / 8);
+            uint4 *dst = reinterpret_cast<uint4 *>(o + ((int64_t)t.l * q_rows + t.qrow + r) * d + (int64_t)t.h * kDh) + c8;
+            *dst = make_uint4(0, 0, 0, 0);
+        }
+    }
+    ChunkIt first;
+    it_first(x, first, u_begin, u_end);
+    if (first.u >= u_end) return;   // uniform across the CTA
+
     if (warp == 0) {
         tmem_alloc(smem_u32(&tmem_slot), kTmemCols);
         tmem_relinquish();
@@ -134,217 +273,388 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
-    // S_c = Q K_c^T into TMEM columns 64 * (c & 1)
-    auto issue_s = [&](int c) {
-        const uint32_t kb = sb + kOffK + 16384u * (c & 1);
-        if (!mbar_wait(bar_k0 + 8 * (c & 1), (c >> 1) & 1, status, &abort_flag, 1)) return;
-        tc_fence_after();
-#pragma unroll
-        for (int kk = 0; kk < 8; ++kk) {
-            const uint32_t koff = (kk >> 2) * 8192u + (kk & 3) * 32u;
-            mma_bf16(tmem + 64u * (c & 1), sdesc_sw128(sb + kOffQ + koff, 16, 1024),
-                     sdesc_sw128(kb + koff, 16, 1024), kIdescS, kk > 0);
+    if (warp == 6) {
+        // ================= TMA producer =================================
+        if (lane == 0) {
+            prefetch_tmap(&tm_q);
+            prefetch_tmap(&tm_k);
+            prefetch_tmap(&tm_r);
+            ChunkIt it = first;
+            uint32_t n = 0, g = 0;
+            int run = -1, pl = -1, ph = -1;
+            auto load_k = [&](const Unit &t, int c) -> bool {
+                const uint32_t ks = g % kKSlots;
+                if (g >= kKSlots && !mbar_wait(B(B_KE + ks), ((g / kKSlots) - 1) & 1, status, &abort_flag, 41))
+                    return false;
+                const uint32_t dst = sb + kOffK + 16384 * ks;
+                mbar_expect_tx(B(B_KF + ks), 16384);
+                tma_load_4d(dst, &tm_k, 0, t.h, t.krow + kChunk * c, t.l, B(B_KF + ks));
+                tma_load_4d(dst + 8192, &tm_k, 64, t.h, t.krow + kChunk * c, t.l, B(B_KF + ks));
+                ++g;
+                return true;
+            };
+            bool ok = true;
+            while (ok && it.u < u_end) {
+                const Unit t = it.t;
+                // keys that fit the ring first (they only wait for older products),
+                // then Q (its slot frees when unit n-2 has its output), then R_h of
+                // a new (layer, head) once the previous run is done, then the rest
+                const int head = min(t.nch, kKSlots);
+                for (int c = 0; c < head && ok; ++c) ok = load_k(t, c);
+                if (!ok) break;
+                const uint32_t qs = n & 1;
+                if (n >= 2 && !mbar_wait(B(B_QE + qs), ((n >> 1) - 1) & 1, status, &abort_flag, 40)) break;
+                mbar_expect_tx(B(B_QF + qs), 16384);
+                tma_load_4d(sb + kOffQ + 16384 * qs, &tm_q, 0, t.h, t.qrow, t.l, B(B_QF + qs));
+                tma_load_4d(sb + kOffQ + 16384 * qs + 8192, &tm_q, 64, t.h, t.qrow, t.l, B(B_QF + qs));
+                if (t.l != pl || t.h != ph) {
+                    ++run;
+                    if (run >= 1 && !mbar_wait(B(B_RE), (run - 1) & 1, status, &abort_flag, 42)) break;
+                    mbar_expect_tx(B(B_RF), 32768);
+                    tma_load_3d(sb + kOffR, &tm_r, 0, 0, t.l * H + t.h, B(B_RF));
+                    tma_load_3d(sb + kOffR + 16384, &tm_r, 64, 0, t.l * H + t.h, B(B_RF));
+                    pl = t.l;
+                    ph = t.h;
+                }
+                for (int c = head; c < t.nch && ok; ++c) ok = load_k(t, c);
+                next_unit(x, it, u_end);
+                ++n;
+            }
         }
-        mma_commit(bar_s0 + 8 * (c & 1));
-    };
-    if (tid == 0) {
-        if (mbar_wait(bar_q, 0, status, &abort_flag, 0)) {
-            issue_s(0);
-            if (nchunks > 1) issue_s(1);
+    } else if (warp == 7) {
+        // ================= MMA issuer (non-blocking over three cursors) ====
+        // tcgen05.mma issue stalls while the tensor pipe is busy, so the work
+        // between products is kept minimal: every shared-memory descriptor is
+        // a base computed here plus a constant (offset / 16 in the start
+        // address field, which cannot carry out of its 14 bits below 256 KB).
+        if (lane == 0) {
+            const uint64_t dq = sdesc_sw128(sb + kOffQ, 16, 1024), dk = sdesc_sw128(sb + kOffK, 16, 1024);
+            const uint64_t dp = sdesc_sw128(sb + kOffP, 16, 1024), dz = sdesc_sw128(sb + kOffZ, 8192, 1024);
+            const uint64_t dr = sdesc_sw128(sb + kOffR, 16, 1024);
+            ChunkIt cs = first, cp = first, co = first;
+            uint32_t gs = 0, ns = 0;   // next S: chunk counter, unit counter
+            uint32_t gp = 0, np = 0;   // next P.Z
+            uint32_t no = 0;           // next output product (unit counter)
+            int run_o = 0;
+            uint32_t idle = 0;
+            while (co.u < u_end && !abort_flag) {
+                bool prog = false;
+                // S of the next chunk: its S buffer is free once P.Z two chunks back
+                // has been issued (that needed the softmax to have read it)
+                if (cs.u < u_end && gs <= gp + 1) {
+                    const uint32_t ks = gs % kKSlots;
+                    const bool qok = cs.c > 0 || mbar_test(B(B_QF + (ns & 1)), (ns >> 1) & 1);
+                    if (qok && mbar_test(B(B_KF + ks), (gs / kKSlots) & 1)) {
+                        tc_fence_after();
+                        const uint64_t qd = dq + 1024u * (ns & 1), kd = dk + 1024u * ks;
+                        const uint32_t sc = tmem + kColS + 64u * (gs & 1);
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t o16 = (kk >> 2) * 512u + (kk & 3) * 2u;   // (kk/4) * 8K + (kk%4) * 32 bytes
+                            mma_bf16(sc, qd + o16, kd + o16, kIdescS, kk > 0);
+                        }
+                        mma_commit(B(B_SF + (gs & 1)));
+                        mma_commit(B(B_KE + ks));
+                        if (it_next(x, cs, u_end)) ++ns;
+                        ++gs;
+                        prog = true;
+                    }
+                }
+                // P.Z of the next chunk; a unit's first one starts its Y buffer
+                // afresh, once the unit two back has had its output read from it
+                if (cp.u < u_end) {
+                    const uint32_t yb = np & 1, b = gp & 1, zs = gp & 3;
+                    const bool yfree = cp.c > 0 || np < 2 || mbar_test(B(B_OE + yb), ((np - 2) >> 1) & 1);
+                    if (yfree && mbar_test(B(B_PF + b), (gp >> 1) & 1) && mbar_test(B(B_ZF + zs), (gp >> 2) & 1)) {
+                        tc_fence_after();
+                        const uint64_t pd = dp + 512u * b, zd = dz + 1024u * zs;
+                        const uint32_t yc = tmem + kColY + 128u * yb;
+                        mma_bf16(yc, pd, zd, kIdescPV, cp.c > 0 ? 1u : 0u);
+#pragma unroll
+                        for (int kk = 1; kk < 4; ++kk)   // P: +32 bytes, Z: +16 kv rows (2 KB) per step
+                            mma_bf16(yc, pd + 2u * kk, zd + 128u * kk, kIdescPV, 1u);
+                        mma_commit(B(B_PV + zs));
+                        if (it_next(x, cp, u_end)) {
+                            mma_commit(B(B_YR + yb));   // the unit's Y is complete
+                            ++np;
+                        }
+                        ++gp;
+                        prog = true;
+                    }
+                }
+                // output product O = Y R_h^T of the oldest unit whose normalised Y is
+                // in shared memory; written over that unit's Y buffer
+                if (np > no) {
+                    if (mbar_test(B(B_YF), no & 1) && mbar_test(B(B_RF), run_o & 1)) {
+                        tc_fence_after();
+                        const uint64_t yd = dq + 1024u * (no & 1);
+                        const uint32_t oc = tmem + kColY + 128u * (no & 1);
+#pragma unroll
+                        for (int kk = 0; kk < 8; ++kk) {
+                            const uint32_t a16 = (kk >> 2) * 512u + (kk & 3) * 2u;    // Y: 8K K-blocks
+                            const uint32_t b16 = (kk >> 2) * 1024u + (kk & 3) * 2u;   // R_h: 16K K-blocks
+                            mma_bf16(oc, yd + a16, dr + b16, kIdescO, kk > 0);
+                        }
+                        mma_commit(B(B_OF));
+                        mma_commit(B(B_QE + (no & 1)));   // Q slot (and the Y in it) free
+                        ChunkIt nx = co;
+                        next_unit(x, nx, u_end);
+                        if (nx.u >= u_end || nx.t.l != co.t.l || nx.t.h != co.t.h) {
+                            mma_commit(B(B_RE));
+                            ++run_o;
+                        }
+                        co = nx;
+                        ++no;
+                        prog = true;
+                    }
+                }
+                if (prog) {
+                    idle = 0;
+                } else if (++idle > (1u << 26)) {
+                    report(status, ROLESUB_ETIMEOUT, 59);
+                    abort_flag = 1;
+                }
+            }
         }
-    }
-
-    float m_run = -INFINITY, l_run = 0.f;
-
-    for (int c = 0; c < nchunks; ++c) {
-        const int buf = c & 1;
-        const int nk = min(kChunk, nc - c * kChunk);
-        if (warp < 2) {
-            mbar_wait(bar_s0 + 8 * buf, (c >> 1) & 1, status, &abort_flag, 2);
-            tc_fence_after();
-            if (tid == 0 && !abort_flag) {
-                // K buffer `buf` is free once S_c completed
-                if (c + 2 < nchunks) {
-                    mbar_expect_tx(bar_k0 + 8 * buf, 16384);
-                    tma_load_4d(sb + kOffK + 16384 * buf, &tm_k, 0, h, krow0 + kChunk * (c + 2), l, bar_k0 + 8 * buf);
-                    tma_load_4d(sb + kOffK + 16384 * buf + 8192, &tm_k, 64, h, krow0 + kChunk * (c + 2), l,
-                                bar_k0 + 8 * buf);
-                }
-                if (c == nchunks - 1) {  // every S MMA is done: R_h replaces both K buffers
-                    mbar_expect_tx(bar_r, 32768);
-                    tma_load_3d(sb + kOffK, &tm_r, 0, 0, l * H + h, bar_r);
-                    tma_load_3d(sb + kOffK + 16384, &tm_r, 64, 0, l * H + h, bar_r);
-                }
+    } else if (warp == 4 || warp == 5) {
+        // ================= value gather (one kv row per thread) ===========
+        // Chunk g goes to Z slot g % 4. Its row record is fetched three chunks
+        // ahead; at iteration g the kept groups of chunk g are copied by
+        // cp.async straight into their swizzled slots of the tile, groups
+        // left over from the slot's previous chunk are zeroed, and the copies
+        // of chunk g - 2 (two commit groups back) are published to the MMA
+        // warp.
+        const int jl = tid - 128;
+        const uint32_t sw = (uint32_t)(jl & 7);
+        // groups of this thread's row that may be non-zero, per Z slot (16 bits
+        // each); a slot's first use clears everything
+        uint64_t dirty = ~0ull;
+        ChunkIt ahead = first, it = first;
+        auto stage_rec = [&](uint32_t gg) {
+            if (ahead.u < u_end) {
+                const int r = ahead.c * kChunk + jl;
+                if (r < ahead.t.nc)
+                    cp_async16(sb + kOffRec + (gg & 3u) * 1024u + (uint32_t)jl * 16u,
+                               rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
             }
-            __syncwarp();
-            // row max of this chunk (scores in the exp2 domain)
-            uint32_t sr[32];
-            float mx = -INFINITY;
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                tmem_ld32(tm_lane(tmem, warp, 64 * buf + 32 * half), sr);
-                tmem_wait_ld();
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (32 * half + j < nk) mx = fmaxf(mx, __uint_as_float(sr[j]) * scale_log2);
+            it_next(x, ahead, u_end);
+            cp_async_commit();
+        };
+        stage_rec(0);
+        stage_rec(1);
+        stage_rec(2);
+        uint32_t g = 0;
+        for (; it.u < u_end && !abort_flag; ++g) {
+            cp_async_wait_group<1>();   // record g and the copies of chunk g - 2 have landed
+            if (g >= 2) {
+                fence_async_smem();
+                mbar_arrive(B(B_ZF + ((g - 2) & 3u)));
             }
-            const float m_new = fmaxf(m_run, mx);
-            const float alpha_c = exp2f(m_run - m_new);
-            float psum = 0.f;
-            uint32_t pk[32];
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                tmem_ld32(tm_lane(tmem, warp, 64 * buf + 32 * half), sr);
-                tmem_wait_ld();
-#pragma unroll
-                for (int j = 0; j < 32; j += 2) {
-                    const int jj = 32 * half + j;
-                    const float p0 = jj < nk ? exp2f(__uint_as_float(sr[j]) * scale_log2 - m_new) : 0.f;
-                    const float p1 = jj + 1 < nk ? exp2f(__uint_as_float(sr[j + 1]) * scale_log2 - m_new) : 0.f;
-                    psum += p0 + p1;
-                    pk[16 * half + j / 2] = pack_bf16(p0, p1);
+            // Z slot g % 4 was last read by the product of chunk g - 4
+            if (g >= 4) mbar_wait(B(B_PV + (g & 3u)), ((g - 4) >> 2) & 1, status, &abort_flag, 60);
+            const int nk = min(kChunk, it.t.nc - it.c * kChunk);
+            uint32_t kept = 0;
+            const uint32_t zrow = sb + kOffZ + 16384u * (g & 3u) + (uint32_t)jl * 128u;
+            if (jl < nk) {
+                const uint4 m = *reinterpret_cast<const uint4 *>(sp + kOffRec + (g & 3u) * 1024u + (uint32_t)jl * 16u);
+                const int k = (int)(m.w >> 27);
+                const uint64_t gid = (uint64_t)m.x | ((uint64_t)m.y << 32);
+                const bf16 *src = packed + (int64_t)it.t.l * packed_per_layer +
+                                  ((int64_t)m.z + (int64_t)it.t.h * (int64_t)(m.w & 0x7FFFFFFu)) * 8;
+                for (int s = 0; s < k; ++s) {
+                    const uint32_t gg = (uint32_t)(gid >> (4 * s)) & 15u;
+                    kept |= 1u << gg;
+                    cp_async16(zrow + (gg >> 3) * 8192u + (((gg & 7u) ^ sw) << 4), src + 8 * s);
                 }
             }
-            l_run = l_run * alpha_c + psum;
-            m_run = m_new;
-            if (c > 0) {
-                // PV_{c-1} is complete (P and Z buffers free); bring the TMEM
-                // accumulator to the new row max before PV_c adds to it
-                mbar_wait(bar_pv, (c - 1) & 1, status, &abort_flag, 3);
+            const uint32_t sh = 16u * (g & 3u);
+            for (uint32_t zm = (uint32_t)(dirty >> sh) & 0xFFFFu & ~kept; zm; zm &= zm - 1) {
+                const uint32_t gg = (uint32_t)(__ffs(zm) - 1);
+                st_shared_v4(zrow + (gg >> 3) * 8192u + (((gg & 7u) ^ sw) << 4), 0, 0, 0, 0);
+            }
+            dirty = (dirty & ~(0xFFFFull << sh)) | ((uint64_t)kept << sh);
+            stage_rec(g + 3);   // also commits this chunk's copies
+            it_next(x, it, u_end);
+        }
+        cp_async_wait_group<0>();
+        fence_async_smem();
+        if (g >= 2) mbar_arrive(B(B_ZF + ((g - 2) & 3u)));
+        if (g >= 1) mbar_arrive(B(B_ZF + ((g - 1) & 3u)));
+    } else if (warp < 4) {
+        // ================= softmax (warps 0-3) ============================
+        // rows ra = 16w + lane/4 and rb = ra + 8 of the unit; column pairs
+        // 8j + 2(lane%4) + {0,1}
+        const int cq = lane & 3;
+        const int ra = 16 * warp + (lane >> 2), rb = ra + 8;
+        const uint32_t lbase = tmem + ((uint32_t)(32 * warp) << 16);
+        ChunkIt it = first;
+        uint32_t n = 0, g = 0;
+        while (it.u < u_end && !abort_flag) {
+            const Unit t = it.t;
+            const uint32_t ycol = kColY + 128u * (n & 1);
+            float ma = -INFINITY, mb = -INFINITY;   // reference maxima (exp2 domain)
+            float la = 0.f, lb = 0.f;               // this thread's share of the row sums
+            for (int c = 0; c < t.nch; ++c, ++g) {
+                const int nk = min(kChunk, t.nc - c * kChunk);
+                mbar_wait(B(B_SF + (g & 1)), (g >> 1) & 1, status, &abort_flag, 70);
                 tc_fence_after();
                 __syncwarp();
-                if (__any_sync(0xffffffffu, alpha_c != 1.f)) {
+                uint32_t sr[32];
+                tmem_ld16x256_x8(lbase + kColS + 64u * (g & 1), sr);
+                tmem_wait_ld();
+                if (nk < kChunk) {
 #pragma unroll
-                    for (int q4 = 0; q4 < 4; ++q4) {
-                        tmem_ld32(tm_lane(tmem, warp, 128 + 32 * q4), sr);
+                    for (int j = 0; j < 8; ++j)
+#pragma unroll
+                        for (int e = 0; e < 2; ++e)
+                            if (8 * j + 2 * cq + e >= nk) {
+                                sr[4 * j + e] = __float_as_uint(-INFINITY);
+                                sr[4 * j + 2 + e] = __float_as_uint(-INFINITY);
+                            }
+                }
+                float xa = -INFINITY, xb = -INFINITY;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    xa = fmaxf(xa, fmaxf(__uint_as_float(sr[4 * j]), __uint_as_float(sr[4 * j + 1])));
+                    xb = fmaxf(xb, fmaxf(__uint_as_float(sr[4 * j + 2]), __uint_as_float(sr[4 * j + 3])));
+                }
+                xa = quad_max(xa) * scale_log2;
+                xb = quad_max(xb) * scale_log2;
+                // raise the reference max (first chunk, or growth beyond 2^8)
+                const bool raise_a = c == 0 || xa > ma + kRescaleLog2;
+                const bool raise_b = c == 0 || xb > mb + kRescaleLog2;
+                const float na = raise_a ? xa : ma, nb = raise_b ? xb : mb;
+                if (c > 0 && __any_sync(0xffffffffu, raise_a || raise_b)) {
+                    const float alpha_a = ex2(ma - na), alpha_b = ex2(mb - nb);
+                    // Y holds chunks up to c-1: wait for the last of them, then rescale
+                    mbar_wait(B(B_PV + ((g - 1) & 3u)), ((g - 1) >> 2) & 1, status, &abort_flag, 71);
+                    tc_fence_after();
+                    __syncwarp();
+                    uint32_t yr[32];
+#pragma unroll 1
+                    for (int h2 = 0; h2 < 2; ++h2) {
+                        const uint32_t ya = lbase + ycol + 64u * h2;
+                        tmem_ld16x256_x8(ya, yr);
                         tmem_wait_ld();
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) sr[j] = __float_as_uint(__uint_as_float(sr[j]) * alpha_c);
-                        tmem_st32(tm_lane(tmem, warp, 128 + 32 * q4), sr);
+                        for (int j = 0; j < 8; ++j) {
+                            yr[4 * j] = __float_as_uint(__uint_as_float(yr[4 * j]) * alpha_a);
+                            yr[4 * j + 1] = __float_as_uint(__uint_as_float(yr[4 * j + 1]) * alpha_a);
+                            yr[4 * j + 2] = __float_as_uint(__uint_as_float(yr[4 * j + 2]) * alpha_b);
+                            yr[4 * j + 3] = __float_as_uint(__uint_as_float(yr[4 * j + 3]) * alpha_b);
+                        }
+                        tmem_st16x256_x8(ya, yr);
                     }
                     tmem_wait_st();
+                    la *= alpha_a;
+                    lb *= alpha_b;
+                }
+                ma = na;
+                mb = nb;
+                uint32_t pa[8], pb[8];
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {   // p = 2^(s * scale - m); masked -inf -> 0
+                    const float a0 = ex2(fmaf(__uint_as_float(sr[4 * j]), scale_log2, -ma));
+                    const float a1 = ex2(fmaf(__uint_as_float(sr[4 * j + 1]), scale_log2, -ma));
+                    const float b0 = ex2(fmaf(__uint_as_float(sr[4 * j + 2]), scale_log2, -mb));
+                    const float b1 = ex2(fmaf(__uint_as_float(sr[4 * j + 3]), scale_log2, -mb));
+                    la += a0 + a1;
+                    lb += b0 + b1;
+                    pa[j] = pack_bf16(a0, a1);
+                    pb[j] = pack_bf16(b0, b1);
+                }
+                // P buffer g & 1 was last read by the product of chunk g - 2
+                if (g >= 2) {
+                    mbar_wait(B(B_PV + ((g - 2) & 3u)), ((g - 2) >> 2) & 1, status, &abort_flag, 72);
+                    tc_fence_after();
+                }
+                const uint32_t pbase = sb + kOffP + 8192u * (g & 1) + 4u * (uint32_t)cq;
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    st_shared_b32(pbase + (uint32_t)ra * 128u + (((uint32_t)j ^ (uint32_t)(ra & 7)) << 4), pa[j]);
+                    st_shared_b32(pbase + (uint32_t)rb * 128u + (((uint32_t)j ^ (uint32_t)(rb & 7)) << 4), pb[j]);
+                }
+                fence_async_smem();
+                tc_fence_before();
+                mbar_arrive(B(B_PF + (g & 1)));
+            }
+            // row sums to the unit tail; buffer n & 1 was last read by the tail
+            // of unit n - 2 before it released that unit's output
+            const float lta = quad_sum(la), ltb = quad_sum(lb);
+            if (n >= 2) mbar_wait(B(B_OE + (n & 1)), ((n - 2) >> 1) & 1, status, &abort_flag, 75);
+            if (cq == 0) {
+                float *lbuf = reinterpret_cast<float *>(sp + kOffL) + 64 * (n & 1);
+                lbuf[ra] = lta;
+                lbuf[rb] = ltb;
+            }
+            mbar_arrive(B(B_LF + (n & 1)));
+            next_unit(x, it, u_end);
+            ++n;
+        }
+    } else {
+        // ================= unit tail (warps 8-11) =========================
+        // y / l -> bf16 operand in the unit's Q slot; after O = Y R_h^T, the
+        // output rows. Lane quadrant w = warp % 4, same row mapping as softmax.
+        const int w = warp & 3, cq = lane & 3;
+        const int ra = 16 * w + (lane >> 2), rb = ra + 8;
+        const uint32_t lbase = tmem + ((uint32_t)(32 * w) << 16);
+        ChunkIt it = first;
+        uint32_t n = 0;
+        while (it.u < u_end) {
+            const Unit t = it.t;
+            const uint32_t yb = n & 1, ycol = kColY + 128u * yb;
+            mbar_wait(B(B_LF + yb), (n >> 1) & 1, status, &abort_flag, 76);
+            const float *lbuf = reinterpret_cast<const float *>(sp + kOffL) + 64 * yb;
+            const float lta = lbuf[ra], ltb = lbuf[rb];
+            mbar_wait(B(B_YR + yb), (n >> 1) & 1, status, &abort_flag, 73);
+            tc_fence_after();
+            __syncwarp();
+            const float ia = lta > 0.f ? 1.f / lta : 0.f, ib = ltb > 0.f ? 1.f / ltb : 0.f;
+            const uint32_t yslot = sb + kOffQ + 16384u * yb + 4u * (uint32_t)cq;
+#pragma unroll 1
+            for (int h2 = 0; h2 < 2; ++h2) {
+                uint32_t yr[32];
+                tmem_ld16x256_x8(lbase + ycol + 64u * h2, yr);
+                tmem_wait_ld();
+                const uint32_t kb = yslot + 8192u * (uint32_t)h2;   // K-block of these 64 columns
+#pragma unroll
+                for (int j = 0; j < 8; ++j) {
+                    st_shared_b32(kb + (uint32_t)ra * 128u + (((uint32_t)j ^ (uint32_t)(ra & 7)) << 4),
+                                  pack_bf16(__uint_as_float(yr[4 * j]) * ia, __uint_as_float(yr[4 * j + 1]) * ia));
+                    st_shared_b32(kb + (uint32_t)rb * 128u + (((uint32_t)j ^ (uint32_t)(rb & 7)) << 4),
+                                  pack_bf16(__uint_as_float(yr[4 * j + 2]) * ib, __uint_as_float(yr[4 * j + 3]) * ib));
                 }
             }
-            // P_c row `tid`: 64 kv = 128 bytes = 8 swizzled 16-byte chunks
-            const uint32_t prow = sb + kOffP + (uint32_t)tid * 128u;
+            fence_async_smem();
+            tc_fence_before();
+            mbar_arrive(B(B_YF));
+            const bool ok = mbar_wait(B(B_OF), n & 1, status, &abort_flag, 74);
+            tc_fence_after();
+            __syncwarp();
+            bf16 *oa = o + ((int64_t)t.l * q_rows + t.qrow + ra) * d + (int64_t)t.h * kDh + 2 * cq;
+            bf16 *ob = oa + 8 * d;
+#pragma unroll 1
+            for (int h2 = 0; h2 < 2; ++h2) {
+                uint32_t orr[32];
+                tmem_ld16x256_x8(lbase + ycol + 64u * h2, orr);
+                tmem_wait_ld();
+                if (ok) {
 #pragma unroll
-            for (int cc = 0; cc < 8; ++cc)
-                st_shared_v4(prow + ((uint32_t)(cc ^ (tid & 7)) << 4), pk[4 * cc], pk[4 * cc + 1], pk[4 * cc + 2],
-                             pk[4 * cc + 3]);
-        } else {
-            // Z_c: kv row jl of the chunk, MN-major (two 64-column blocks)
-            if (c > 0) mbar_wait(bar_pv, (c - 1) & 1, status, &abort_flag, 4);
-            const int jl = tid - 64;
-            const int j = c * kChunk + jl;
-            const uint32_t zrow = sb + kOffZ + (uint32_t)jl * 128u;
-            const uint32_t sw = (uint32_t)(jl & 7);
-            uint32_t kept = 0;
-            if (j < nc) {
-                int m = 0;
-                while (m < ROLESUB_NUM_KINDS - 1 && j >= row0[m + 1]) ++m;
-                const int k = sg[m].k;
-                const int64_t ti = j - row0[m];
-                const uint8_t *ix = idx + (int64_t)l * idx_per_layer + sg[m].idx_off + ti * k;
-                const uint4 *src = reinterpret_cast<const uint4 *>(
-                    packed + (int64_t)l * packed_per_layer + sg[m].packed_off + ((int64_t)h * sg[m].n_tokens + ti) * k * 8);
-                int gid[kG];
-#pragma unroll
-                for (int s = 0; s < kG; ++s)
-                    if (s < k) gid[s] = ix[s];
-#pragma unroll
-                for (int s = 0; s < kG; ++s) {
-                    if (s < k) {
-                        const int g = gid[s];
-                        if (g >= kG) {
-                            report(status, ROLESUB_EDEVICE, (int)(ep.row_begin + j));
-                            continue;
-                        }
-                        if ((kept >> g) & 1u) continue;   // repeated index: keep the first
-                        kept |= 1u << g;
-                        cp_async16(zrow + (uint32_t)(g >> 3) * 8192u + (((uint32_t)(g & 7) ^ sw) << 4), src + s);
+                    for (int j = 0; j < 8; ++j) {
+                        const int col = 64 * h2 + 8 * j;
+                        if (ra < t.nq)
+                            *reinterpret_cast<uint32_t *>(oa + col) =
+                                pack_bf16(__uint_as_float(orr[4 * j]), __uint_as_float(orr[4 * j + 1]));
+                        if (rb < t.nq)
+                            *reinterpret_cast<uint32_t *>(ob + col) =
+                                pack_bf16(__uint_as_float(orr[4 * j + 2]), __uint_as_float(orr[4 * j + 3]));
                     }
                 }
             }
-#pragma unroll
-            for (int g = 0; g < kG; ++g)
-                if (!((kept >> g) & 1u))
-                    st_shared_v4(zrow + (uint32_t)(g >> 3) * 8192u + (((uint32_t)(g & 7) ^ sw) << 4), 0, 0, 0, 0);
-            cp_async_wait_all();
-        }
-        fence_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-        if (tid == 0 && !abort_flag) {
-            // Y_c = P_c Z_c (fresh accumulator), then the next S on this buffer
-#pragma unroll
-            for (int kk = 0; kk < 4; ++kk)
-                mma_bf16(tmem + 128, sdesc_sw128(sb + kOffP + 32u * kk, 16, 1024),
-                         sdesc_sw128(sb + kOffZ + 2048u * kk, 8192, 1024), kIdescPV, (c > 0 || kk > 0) ? 1u : 0u);
-            mma_commit(bar_pv);
-            if (c + 2 < nchunks) issue_s(c + 2);
-        }
-    }
-
-    if (warp < 2) {
-        mbar_wait(bar_pv, (nchunks - 1) & 1, status, &abort_flag, 5);
-        tc_fence_after();
-        __syncwarp();
-        uint32_t sr[32];
-        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-        // y / l as the bf16 A operand (Q region: K-blocks of 64 columns at +0, +8K)
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-            tmem_ld32(tm_lane(tmem, warp, 128 + 32 * q4), sr);
-            tmem_wait_ld();
-#pragma unroll
-            for (int c4 = 0; c4 < 4; ++c4) {
-                const int cc = 4 * q4 + c4;   // 16-byte chunk (8 columns) of the 128-column row
-                const uint32_t addr = sb + kOffQ + (uint32_t)(cc >> 3) * 8192u + (uint32_t)tid * 128u +
-                                      ((uint32_t)((cc & 7) ^ (tid & 7)) << 4);
-                const float *f = reinterpret_cast<const float *>(sr) + 8 * c4;
-                st_shared_v4(addr, pack_bf16(f[0] * inv, f[1] * inv), pack_bf16(f[2] * inv, f[3] * inv),
-                             pack_bf16(f[4] * inv, f[5] * inv), pack_bf16(f[6] * inv, f[7] * inv));
-            }
-        }
-    }
-    fence_async_smem();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (tid == 0 && !abort_flag) {
-        // O = Y R_h^T: B = R_h rows (output dim) x K-major columns
-        if (mbar_wait(bar_r, 0, status, &abort_flag, 6)) {
-            tc_fence_after();
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-                const uint32_t aoff = (kk >> 2) * 8192u + (kk & 3) * 32u;
-                const uint32_t boff = (kk >> 2) * 16384u + (kk & 3) * 32u;
-                mma_bf16(tmem, sdesc_sw128(sb + kOffQ + aoff, 16, 1024), sdesc_sw128(sb + kOffK + boff, 16, 1024),
-                         kIdescO, kk > 0);
-            }
-            mma_commit(bar_o);
-        }
-    }
-    if (warp < 2) {
-        const bool ok = mbar_wait(bar_o, 0, status, &abort_flag, 7);
-        tc_fence_after();
-        __syncwarp();
-        bf16 *orow = o + ((int64_t)l * q_rows + ep.q_row_begin + qb + tid) * d + (int64_t)h * kDh;
-        uint32_t sr[32];
-#pragma unroll
-        for (int q4 = 0; q4 < 4; ++q4) {
-            tmem_ld32(tm_lane(tmem, warp, 32 * q4), sr);
-            tmem_wait_ld();
-            if (ok && tid < nq) {
-                uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * q4);
-#pragma unroll
-                for (int v4 = 0; v4 < 4; ++v4)
-                    dst[v4] = make_uint4(pack_bf16(__uint_as_float(sr[8 * v4]), __uint_as_float(sr[8 * v4 + 1])),
-                                         pack_bf16(__uint_as_float(sr[8 * v4 + 2]), __uint_as_float(sr[8 * v4 + 3])),
-                                         pack_bf16(__uint_as_float(sr[8 * v4 + 4]), __uint_as_float(sr[8 * v4 + 5])),
-                                         pack_bf16(__uint_as_float(sr[8 * v4 + 6]), __uint_as_float(sr[8 * v4 + 7])));
-            }
+            tc_fence_before();
+            mbar_arrive(B(B_OE + yb));
+            next_unit(x, it, u_end);
+            ++n;
         }
     }
     tc_fence_before();
@@ -368,6 +678,7 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
     const rolesub_plan &P = *a.plan.hdr;
     if (P.max_query_tokens == 0 || P.num_episodes == 0) return cudaSuccess;
     const int H = S.num_heads, L = S.num_layers;
+    const int64_t rows = P.rows_per_layer;
     CUtensorMap tq, tk, tr;
     {
         const uint64_t dims[4] = {(uint64_t)kDh, (uint64_t)H, (uint64_t)P.q_rows_per_layer, (uint64_t)L};
@@ -376,7 +687,7 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
         if (!make_bf16_map(&tq, a.q, 4, dims, str, box)) return cudaErrorInvalidValue;
     }
     {
-        const uint64_t dims[4] = {(uint64_t)kDh, (uint64_t)H, (uint64_t)P.rows_per_layer, (uint64_t)L};
+        const uint64_t dims[4] = {(uint64_t)kDh, (uint64_t)H, (uint64_t)rows, (uint64_t)L};
         const uint64_t str[3] = {(uint64_t)a.k_hs * 2, (uint64_t)a.k_rs * 2, (uint64_t)a.k_ls * 2};
         const uint32_t box[4] = {64, 1, (uint32_t)kChunk, 1};
         if (!make_bf16_map(&tk, a.K, 4, dims, str, box)) return cudaErrorInvalidValue;
@@ -389,14 +700,29 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
     }
     cudaError_t err = cudaFuncSetAttribute(k_attend_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (err != cudaSuccess) return err;
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+        sms = 152;
+    // per-row records (kept groups, packed offset) from the caller's indices
+    uint4 *recs = reinterpret_cast<uint4 *>(a.ws.row_store);
+    err = launch_row_store(a.plan, L, const_cast<uint8_t *>(a.idx), P.idx_bytes_per_layer, false, recs, a.ws.status,
+                           a.stream);
+    if (err != cudaSuccess) return err;
     const int qtiles = (P.max_query_tokens + kQRows - 1) / kQRows;
-    PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev};
     const float scale = a.scale > 0.f ? a.scale : 1.0f / sqrtf((float)kDh);
-    k_attend_tc<<<dim3(H, P.num_episodes * qtiles, L), kThreads, kSmemBytes, a.stream>>>(
-        tq, tk, tr, (const bf16 *)a.packed, P.packed_elems_per_layer, a.idx, P.idx_bytes_per_layer, pd, H, qtiles,
-        P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o, a.ws.status);
-    count_launches(1);
-    return cudaGetLastError();
+    for (int e0 = 0; e0 < P.num_episodes; e0 += kMaxEp) {
+        const int E = std::min(kMaxEp, P.num_episodes - e0);
+        const int64_t units = (int64_t)L * H * E * qtiles;
+        const int grid = (int)std::min<int64_t>(units, sms);
+        k_attend_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(
+            tq, tk, tr, (const bf16 *)a.packed, P.packed_elems_per_layer, recs, rows, a.plan.eps_dev, e0, E, H, L,
+            qtiles, P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o, a.ws.status);
+        count_launches(1);
+        err = cudaGetLastError();
+        if (err != cudaSuccess) return err;
+    }
+    return cudaSuccess;
 }
 
 }  // namespace rs

@@ -50,8 +50,9 @@ constexpr uint32_t kIdesc = idesc_bf16(128, 128, true);
 //   z:    (packed_off + i * k * d_s) / 8, the row's first group for head 0
 //   w:    k << 27 | n * k, i.e. kept groups and the per-head stride / 8
 // k = 0 means nothing is stored for the row (or its indices were corrupt).
+// write_identity: also write indices 0..S-1 of k = S rows (compress only).
 __global__ void __launch_bounds__(256)
-k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_per_layer,
+k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_per_layer, bool write_identity,
             uint4 *__restrict__ meta, int32_t *status)
 {
     const int l = blockIdx.y;
@@ -65,7 +66,8 @@ k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_p
     int kk = k;
     if (k == kG) {
         gid = 0xFEDCBA9876543210ull;
-        for (int s = 0; s < kG; ++s) ix[s] = (uint8_t)s;   // byte stores: no alignment needed
+        if (write_identity)
+            for (int s = 0; s < kG; ++s) ix[s] = (uint8_t)s;   // byte stores: no alignment needed
     } else {
         for (int s = 0; s < k; ++s) {
             const uint32_t g = ix[s];
@@ -258,14 +260,24 @@ cudaError_t launch_rotate_tc(const CompressArgs &a)
     while ((int64_t)H * L * splits < 4 * 152 && splits < ntiles) ++splits;
     const int per = (ntiles + splits - 1) / splits;
     splits = (ntiles + per - 1) / per;
-    PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev,
-               a.plan.route_tiles_dev};
     uint4 *meta = reinterpret_cast<uint4 *>(a.ws.row_store);
-    k_row_store<<<dim3((unsigned)((rows + 255) / 256), L), 256, 0, a.stream>>>(pd, rows, a.idx,
-                                                                              P.idx_bytes_per_layer, meta, a.ws.status);
+    err = launch_row_store(a.plan, L, a.idx, P.idx_bytes_per_layer, true, meta, a.ws.status, a.stream);
+    if (err != cudaSuccess) return err;
     k_rotate_tc<<<dim3(H, L, splits), kThreads, kSmemBytes, a.stream>>>(
         tv, tr, meta, rows, H, per, ntiles, (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
-    count_launches(2);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_row_store(const PlanView &pv, int L, uint8_t *idx, int64_t idx_per_layer, bool write_identity,
+                             uint4 *recs, int32_t *status, cudaStream_t stream)
+{
+    const int64_t rows = pv.hdr->rows_per_layer;
+    if (rows == 0) return cudaSuccess;
+    PlanDev pd{pv.segs_dev, pv.eps_dev, pv.row_seg_dev, pv.routed_dev, pv.stored_dev, pv.route_tiles_dev};
+    k_row_store<<<dim3((unsigned)((rows + 255) / 256), L), 256, 0, stream>>>(pd, rows, idx, idx_per_layer,
+                                                                            write_identity, recs, status);
+    count_launches(1);
     return cudaGetLastError();
 }
 

@@ -154,6 +154,33 @@ def test_bad_stored_index_is_reported_not_trapped():
     assert rs.device_status() == (0, 0)
 
 
+def test_bad_stored_index_bf16_tensor_core_path():
+    import parity
+    wl = synth.c1()
+    inp = synth.gen_inputs(wl)
+    gpu = parity.run_gpu(wl, inp)
+    rs = gpu["rs"]
+    idx = gpu["idx"].copy()
+    idx[0, 4 * 7 + 2] = 99                 # vis token 7 (k = 4): group id >= S
+    o = rs.attend(parity.to_torch(inp["q"], wl.dtype), parity.to_torch(inp["K"], wl.dtype),
+                  parity.to_torch(gpu["packed"], wl.dtype), parity.to_torch(idx, wl.dtype),
+                  parity.to_torch(inp["R"], wl.dtype))
+    code, detail = rs.device_status()
+    assert code == 4 and detail == 7
+    assert np.all(np.isfinite(synth.widen(parity.from_torch(o, wl.dtype), wl.dtype)))
+    from paper_2608_18410_gb300 import rolesub
+    rolesub.rolesub_reset_device_status(rs.workspace)
+
+
+def test_many_small_episodes_bf16():
+    """More episodes than one attention launch covers (episode table limit)."""
+    rng = np.random.default_rng(5)
+    eps = [synth.Episode(int(rng.integers(0, 5)), int(rng.integers(0, 3)), int(rng.integers(0, 3)),
+                         int(rng.choice([1, 2, 16])), int(rng.choice([0, 4, 16]))) for _ in range(600)]
+    wl = _wl("bf16", eps, L=1, H=2, C=64, F=256)
+    _run(wl, [(0, e) for e in (0, 1, 255, 511, 512, 513, 599)])
+
+
 def test_repeated_calls_are_deterministic():
     import parity
     wl = synth.c1()
