@@ -76,7 +76,7 @@ constexpr int kChunk = 64;   // cache tokens per chunk
 constexpr int kQRows = 64;   // query rows per unit
 constexpr int kDh = 128;
 constexpr int kG = 16;       // groups per head (d_s = 8)
-constexpr int kMaxEp = 256;  // episodes per launch (episode table in smem)
+constexpr int kMaxUnits = 448;   // units per CTA and launch (unit list in smem)
 constexpr int kKSlots = 4;
 constexpr float kRescaleLog2 = 8.f;   // raise the reference max beyond 2^8 growth
 
@@ -88,8 +88,8 @@ constexpr uint32_t kOffZ = 147456;                   // 4 x 16K ring
 constexpr int kZSlots = 4;
 constexpr uint32_t kOffRec = kOffZ + kZSlots * 16384; // 4 x 64 x 16 B
 constexpr uint32_t kOffL = kOffRec + 4096;           // 2 x 64 fp32 row sums
-constexpr uint32_t kOffEp = kOffL + 1024;            // 4 x kMaxEp int32
-constexpr uint32_t kOffBar = kOffEp + 16 * kMaxEp;
+constexpr uint32_t kOffUnits = kOffL + 1024;         // kMaxUnits x 16 B unit records
+constexpr uint32_t kOffBar = kOffUnits + 16 * kMaxUnits;
 constexpr uint32_t kSmemBytes = kOffBar + 512 + 1024;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColS = 0, kColY = 128;   // Y[b] at kColY + 128b
@@ -105,90 +105,54 @@ enum {
 };
 
 struct Unit {
-    int l, h, e, nq, nc, nch, krow, qrow;
+    int l, h, nq, nc, nch, krow, qrow;
 };
 
-struct Ctx {
-    const int *ep_row, *ep_qrow, *ep_nc, *ep_nq;  // shared-memory episode table
-    int H, E, qtiles;
-};
+// A CTA's units with queries and cache tokens, in processing order, as
+// 16-byte records {first cache row, first query row, n_cache,
+// n_q | h << 8 | l << 18} built once at kernel start; every role walks the
+// same list.
+__device__ __forceinline__ Unit load_unit(const uint8_t *sp, int k)
+{
+    const uint4 v = *reinterpret_cast<const uint4 *>(sp + kOffUnits + 16u * (uint32_t)k);
+    Unit t;
+    t.krow = (int)v.x;
+    t.qrow = (int)v.y;
+    t.nc = (int)v.z;
+    t.nch = (t.nc + kChunk - 1) / kChunk;
+    t.nq = (int)(v.w & 255u);
+    t.h = (int)((v.w >> 8) & 1023u);
+    t.l = (int)(v.w >> 18);
+    return t;
+}
 
-// Iterator over a CTA's units -- (layer, head, episode, query tile), query
-// tiles fastest, then episodes -- and over the chunks of each unit. Units
-// advance by counters (no division), so the iterator stays small wherever it
-// is inlined.
+// Iterator over the units of the list and the chunks of each unit.
 struct ChunkIt {
-    int u, c, qt;   // unit index (u_end = done), chunk within unit, query tile
+    int k, c;   // unit (nu = done), chunk within unit
     Unit t;
 };
 
-__device__ __forceinline__ void fill(const Ctx &x, ChunkIt &it)
+__device__ __forceinline__ void it_first(const uint8_t *sp, ChunkIt &it, int nu)
 {
-    const int e = it.t.e, qb = it.qt * kQRows;
-    it.t.nq = max(0, min(kQRows, x.ep_nq[e] - qb));
-    it.t.nc = x.ep_nc[e];
-    it.t.nch = (it.t.nc + kChunk - 1) / kChunk;
-    it.t.krow = x.ep_row[e];
-    it.t.qrow = x.ep_qrow[e] + qb;
-}
-
-__device__ __forceinline__ void seek(const Ctx &x, ChunkIt &it, int u)
-{
-    it.u = u;
+    it.k = 0;
     it.c = 0;
-    it.qt = u % x.qtiles;
-    int r = u / x.qtiles;
-    it.t.e = r % x.E;
-    r /= x.E;
-    it.t.h = r % x.H;
-    it.t.l = r / x.H;
-    fill(x, it);
-}
-
-__device__ __forceinline__ void step(const Ctx &x, ChunkIt &it)
-{
-    ++it.u;
-    if (++it.qt == x.qtiles) {
-        it.qt = 0;
-        if (++it.t.e == x.E) {
-            it.t.e = 0;
-            if (++it.t.h == x.H) {
-                it.t.h = 0;
-                ++it.t.l;
-            }
-        }
-    }
-    fill(x, it);
-}
-
-__device__ __forceinline__ bool busy(const Unit &t) { return t.nq > 0 && t.nc > 0; }
-
-__device__ __forceinline__ void skip_idle(const Ctx &x, ChunkIt &it, int u_end)
-{
-    while (it.u < u_end && !busy(it.t)) step(x, it);
-}
-
-__device__ __forceinline__ void it_first(const Ctx &x, ChunkIt &it, int u_begin, int u_end)
-{
-    seek(x, it, u_begin);
-    skip_idle(x, it, u_end);
+    if (nu > 0) it.t = load_unit(sp, 0);
 }
 
 // advances one chunk; returns true when it moved to another unit
-__device__ __forceinline__ bool it_next(const Ctx &x, ChunkIt &it, int u_end)
+__device__ __forceinline__ bool it_next(const uint8_t *sp, ChunkIt &it, int nu)
 {
-    if (it.u >= u_end) return false;
+    if (it.k >= nu) return false;
     if (++it.c < it.t.nch) return false;
     it.c = 0;
-    step(x, it);
-    skip_idle(x, it, u_end);
+    if (++it.k < nu) it.t = load_unit(sp, it.k);
     return true;
 }
 
-__device__ __forceinline__ void next_unit(const Ctx &x, ChunkIt &it, int u_end)
+__device__ __forceinline__ void next_unit(const uint8_t *sp, ChunkIt &it, int nu)
 {
-    it.c = it.t.nch - 1;
-    it_next(x, it, u_end);
+    it.c = 0;
+    if (++it.k < nu) it.t = load_unit(sp, it.k);
 }
 
 __device__ __forceinline__ float quad_sum(float v)
@@ -207,7 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
             const __grid_constant__ CUtensorMap tm_r, const bf16 *__restrict__ packed,
             int64_t packed_per_layer, const uint4 *__restrict__ rec, int64_t rows,
-            const rolesub_episode *__restrict__ eps, int e0, int E, int H, int L, int qtiles, int64_t q_rows,
+            const rolesub_episode *__restrict__ eps, int E, int H, int qtiles, int64_t u0, int64_t u1, int64_t q_rows,
             float scale_log2, bf16 *__restrict__ o, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -219,20 +183,10 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int64_t d = (int64_t)H * kDh;
 
-    // ---- episode table and unit range ------------------------------------
-    int *ep_tab = reinterpret_cast<int *>(sp + kOffEp);
-    for (int i = tid; i < E; i += kThreads) {
-        const rolesub_episode ep = eps[e0 + i];
-        ep_tab[i] = (int)ep.row_begin;
-        ep_tab[kMaxEp + i] = (int)ep.q_row_begin;
-        ep_tab[2 * kMaxEp + i] = ep.n_cache;
-        ep_tab[3 * kMaxEp + i] = ep.n_query;
-    }
-    const Ctx x{ep_tab, ep_tab + kMaxEp, ep_tab + 2 * kMaxEp, ep_tab + 3 * kMaxEp, H, E, qtiles};
-    const int64_t U = (int64_t)L * H * E * qtiles;
-    const int u_begin = (int)(U * blockIdx.x / gridDim.x);
-    const int u_end = (int)(U * (blockIdx.x + 1) / gridDim.x);
-
+    // ---- this CTA's share of units [u0, u1) -------------------------------
+    const int64_t span = u1 - u0;
+    const int64_t ub = u0 + span * blockIdx.x / gridDim.x;
+    const int cnt = (int)(u0 + span * (blockIdx.x + 1) / gridDim.x - ub);   // <= kMaxUnits
     const uint32_t bar = sb + kOffBar;
     auto B = [&](int i) { return bar + 8u * (uint32_t)i; };
     if (tid == 0) {
@@ -248,21 +202,50 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
     }
     __syncthreads();
 
-    // units without cache tokens: o = 0
-    ChunkIt z;
-    seek(x, z, u_begin);
-    for (; z.u < u_end; step(x, z)) {
-        const Unit &t = z.t;
-        if (t.nq == 0 || t.nc > 0) continue;
-        for (int i = tid; i < t.nq * (kDh / 8); i += kThreads) {
-            const int r = i / (kDh / 8), c8 = i % (kDh / 8);
-            uint4 *dst = reinterpret_cast<uint4 *>(o + ((int64_t)t.l * q_rows + t.qrow + r) * d + (int64_t)t.h * kDh) + c8;
-            *dst = make_uint4(0, 0, 0, 0);
+    // unit list: units with queries and cache tokens, in order; units with
+    // queries but no cache tokens get o = 0 here
+    __shared__ int warp_cnt[kThreads / 32];
+    int nu = 0;
+    for (int base = 0; base < cnt; base += kThreads) {
+        const int i = base + tid;
+        bool keep = false;
+        uint4 rec4 = make_uint4(0, 0, 0, 0);
+        if (i < cnt) {
+            const int64_t u = ub + i;
+            const int qt = (int)(u % qtiles);
+            int64_t r = u / qtiles;
+            const int e = (int)(r % E);
+            r /= E;
+            const int h = (int)(r % H), l = (int)(r / H);
+            const rolesub_episode ep = eps[e];
+            const int nq = max(0, min(kQRows, ep.n_query - qt * kQRows));
+            const int qrow = (int)ep.q_row_begin + qt * kQRows;
+            keep = nq > 0 && ep.n_cache > 0;
+            rec4 = make_uint4((uint32_t)ep.row_begin, (uint32_t)qrow, (uint32_t)ep.n_cache,
+                              (uint32_t)nq | ((uint32_t)h << 8) | ((uint32_t)l << 18));
+            if (nq > 0 && ep.n_cache == 0)
+                for (int j = 0; j < nq * (kDh / 8); ++j) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(o + ((int64_t)l * q_rows + qrow + j / (kDh / 8)) * d +
+                                                           (int64_t)h * kDh) + j % (kDh / 8);
+                    *dst = make_uint4(0, 0, 0, 0);
+                }
         }
+        const uint32_t bal = __ballot_sync(0xffffffffu, keep);
+        if (lane == 0) warp_cnt[warp] = __popc(bal);
+        __syncthreads();
+        int off = nu, tot = 0;
+        for (int w = 0; w < kThreads / 32; ++w) {
+            off += w < warp ? warp_cnt[w] : 0;
+            tot += warp_cnt[w];
+        }
+        if (keep)
+            *reinterpret_cast<uint4 *>(sp + kOffUnits + 16u * (uint32_t)(off + __popc(bal & ((1u << lane) - 1u)))) = rec4;
+        nu += tot;
+        __syncthreads();
     }
+    if (nu == 0) return;   // uniform across the CTA
     ChunkIt first;
-    it_first(x, first, u_begin, u_end);
-    if (first.u >= u_end) return;   // uniform across the CTA
+    it_first(sp, first, nu);
 
     if (warp == 0) {
         tmem_alloc(smem_u32(&tmem_slot), kTmemCols);
@@ -294,7 +277,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 return true;
             };
             bool ok = true;
-            while (ok && it.u < u_end) {
+            while (ok && it.k < nu) {
                 const Unit t = it.t;
                 // keys that fit the ring first (they only wait for older products),
                 // then Q (its slot frees when unit n-2 has its output), then R_h of
@@ -317,7 +300,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                     ph = t.h;
                 }
                 for (int c = head; c < t.nch && ok; ++c) ok = load_k(t, c);
-                next_unit(x, it, u_end);
+                next_unit(sp, it, nu);
                 ++n;
             }
         }
@@ -337,11 +320,11 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             uint32_t no = 0;           // next output product (unit counter)
             int run_o = 0;
             uint32_t idle = 0;
-            while (co.u < u_end && !abort_flag) {
+            while (co.k < nu && !abort_flag) {
                 bool prog = false;
                 // S of the next chunk: its S buffer is free once P.Z two chunks back
                 // has been issued (that needed the softmax to have read it)
-                if (cs.u < u_end && gs <= gp + 1) {
+                if (cs.k < nu && gs <= gp + 1) {
                     const uint32_t ks = gs % kKSlots;
                     const bool qok = cs.c > 0 || mbar_test(B(B_QF + (ns & 1)), (ns >> 1) & 1);
                     if (qok && mbar_test(B(B_KF + ks), (gs / kKSlots) & 1)) {
@@ -355,14 +338,14 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                         }
                         mma_commit(B(B_SF + (gs & 1)));
                         mma_commit(B(B_KE + ks));
-                        if (it_next(x, cs, u_end)) ++ns;
+                        if (it_next(sp, cs, nu)) ++ns;
                         ++gs;
                         prog = true;
                     }
                 }
                 // P.Z of the next chunk; a unit's first one starts its Y buffer
                 // afresh, once the unit two back has had its output read from it
-                if (cp.u < u_end) {
+                if (cp.k < nu) {
                     const uint32_t yb = np & 1, b = gp & 1, zs = gp & 3;
                     const bool yfree = cp.c > 0 || np < 2 || mbar_test(B(B_OE + yb), ((np - 2) >> 1) & 1);
                     if (yfree && mbar_test(B(B_PF + b), (gp >> 1) & 1) && mbar_test(B(B_ZF + zs), (gp >> 2) & 1)) {
@@ -374,7 +357,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                         for (int kk = 1; kk < 4; ++kk)   // P: +32 bytes, Z: +16 kv rows (2 KB) per step
                             mma_bf16(yc, pd + 2u * kk, zd + 128u * kk, kIdescPV, 1u);
                         mma_commit(B(B_PV + zs));
-                        if (it_next(x, cp, u_end)) {
+                        if (it_next(sp, cp, nu)) {
                             mma_commit(B(B_YR + yb));   // the unit's Y is complete
                             ++np;
                         }
@@ -398,8 +381,8 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                         mma_commit(B(B_OF));
                         mma_commit(B(B_QE + (no & 1)));   // Q slot (and the Y in it) free
                         ChunkIt nx = co;
-                        next_unit(x, nx, u_end);
-                        if (nx.u >= u_end || nx.t.l != co.t.l || nx.t.h != co.t.h) {
+                        next_unit(sp, nx, nu);
+                        if (nx.k >= nu || nx.t.l != co.t.l || nx.t.h != co.t.h) {
                             mma_commit(B(B_RE));
                             ++run_o;
                         }
@@ -431,20 +414,20 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         uint64_t dirty = ~0ull;
         ChunkIt ahead = first, it = first;
         auto stage_rec = [&](uint32_t gg) {
-            if (ahead.u < u_end) {
+            if (ahead.k < nu) {
                 const int r = ahead.c * kChunk + jl;
                 if (r < ahead.t.nc)
                     cp_async16(sb + kOffRec + (gg & 3u) * 1024u + (uint32_t)jl * 16u,
                                rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
             }
-            it_next(x, ahead, u_end);
+            it_next(sp, ahead, nu);
             cp_async_commit();
         };
         stage_rec(0);
         stage_rec(1);
         stage_rec(2);
         uint32_t g = 0;
-        for (; it.u < u_end && !abort_flag; ++g) {
+        for (; it.k < nu && !abort_flag; ++g) {
             cp_async_wait_group<1>();   // record g and the copies of chunk g - 2 have landed
             if (g >= 2) {
                 fence_async_smem();
@@ -474,7 +457,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             }
             dirty = (dirty & ~(0xFFFFull << sh)) | ((uint64_t)kept << sh);
             stage_rec(g + 3);   // also commits this chunk's copies
-            it_next(x, it, u_end);
+            it_next(sp, it, nu);
         }
         cp_async_wait_group<0>();
         fence_async_smem();
@@ -489,7 +472,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         const uint32_t lbase = tmem + ((uint32_t)(32 * warp) << 16);
         ChunkIt it = first;
         uint32_t n = 0, g = 0;
-        while (it.u < u_end && !abort_flag) {
+        while (it.k < nu && !abort_flag) {
             const Unit t = it.t;
             const uint32_t ycol = kColY + 128u * (n & 1);
             float ma = -INFINITY, mb = -INFINITY;   // reference maxima (exp2 domain)
@@ -588,7 +571,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 lbuf[rb] = ltb;
             }
             mbar_arrive(B(B_LF + (n & 1)));
-            next_unit(x, it, u_end);
+            next_unit(sp, it, nu);
             ++n;
         }
     } else {
@@ -600,7 +583,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         const uint32_t lbase = tmem + ((uint32_t)(32 * w) << 16);
         ChunkIt it = first;
         uint32_t n = 0;
-        while (it.u < u_end) {
+        while (it.k < nu) {
             const Unit t = it.t;
             const uint32_t yb = n & 1, ycol = kColY + 128u * yb;
             mbar_wait(B(B_LF + yb), (n >> 1) & 1, status, &abort_flag, 76);
@@ -653,7 +636,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             }
             tc_fence_before();
             mbar_arrive(B(B_OE + yb));
-            next_unit(x, it, u_end);
+            next_unit(sp, it, nu);
             ++n;
         }
     }
@@ -669,7 +652,9 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
 
 bool attend_tc_supported(const rolesub_shape *s)
 {
-    return s->dtype == ROLESUB_BF16 && s->head_dim == kDh && s->num_groups == kG;
+    // unit records hold h in 10 bits and l in 14
+    return s->dtype == ROLESUB_BF16 && s->head_dim == kDh && s->num_groups == kG && s->num_heads <= 1024 &&
+           s->num_layers <= 16384;
 }
 
 cudaError_t launch_attend_tc(const AttendArgs &a)
@@ -711,13 +696,16 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
     if (err != cudaSuccess) return err;
     const int qtiles = (P.max_query_tokens + kQRows - 1) / kQRows;
     const float scale = a.scale > 0.f ? a.scale : 1.0f / sqrtf((float)kDh);
-    for (int e0 = 0; e0 < P.num_episodes; e0 += kMaxEp) {
-        const int E = std::min(kMaxEp, P.num_episodes - e0);
-        const int64_t units = (int64_t)L * H * E * qtiles;
-        const int grid = (int)std::min<int64_t>(units, sms);
+    // units (layer, head, episode, query tile); a launch gives each CTA at
+    // most kMaxUnits of them
+    const int E = P.num_episodes;
+    const int64_t U = (int64_t)L * H * E * qtiles, per_launch = (int64_t)kMaxUnits * sms;
+    for (int64_t u0 = 0; u0 < U; u0 += per_launch) {
+        const int64_t u1 = std::min(U, u0 + per_launch);
+        const int grid = (int)std::min<int64_t>(u1 - u0, sms);
         k_attend_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(
-            tq, tk, tr, (const bf16 *)a.packed, P.packed_elems_per_layer, recs, rows, a.plan.eps_dev, e0, E, H, L,
-            qtiles, P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o, a.ws.status);
+            tq, tk, tr, (const bf16 *)a.packed, P.packed_elems_per_layer, recs, rows, a.plan.eps_dev, E, H, qtiles,
+            u0, u1, P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o, a.ws.status);
         count_launches(1);
         err = cudaGetLastError();
         if (err != cudaSuccess) return err;
