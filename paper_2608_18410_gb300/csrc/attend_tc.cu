@@ -551,12 +551,15 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                     mbar_wait(B(B_PV + ((g - 2) & 3u)), ((g - 2) >> 2) & 1, status, &abort_flag, 72);
                     tc_fence_after();
                 }
-                const uint32_t pbase = sb + kOffP + 8192u * (g & 1) + 4u * (uint32_t)cq;
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    st_shared_b32(pbase + (uint32_t)ra * 128u + (((uint32_t)j ^ (uint32_t)(ra & 7)) << 4), pa[j]);
-                    st_shared_b32(pbase + (uint32_t)rb * 128u + (((uint32_t)j ^ (uint32_t)(rb & 7)) << 4), pb[j]);
-                }
+                // 8x8 blocks (rows of ra / rb, 8 columns = one swizzle chunk each):
+                // lane t addresses row t%8 of block t/8
+                const uint32_t prow = sb + kOffP + 8192u * (g & 1) + (uint32_t)(16 * warp + (lane & 7)) * 128u;
+                const uint32_t c0 = ((uint32_t)(lane >> 3) ^ (uint32_t)(lane & 7)) << 4;
+                const uint32_t c1 = ((uint32_t)((lane >> 3) + 4) ^ (uint32_t)(lane & 7)) << 4;
+                stmatrix_x4(prow + c0, pa[0], pa[1], pa[2], pa[3]);
+                stmatrix_x4(prow + c1, pa[4], pa[5], pa[6], pa[7]);
+                stmatrix_x4(prow + 1024u + c0, pb[0], pb[1], pb[2], pb[3]);
+                stmatrix_x4(prow + 1024u + c1, pb[4], pb[5], pb[6], pb[7]);
                 fence_async_smem();
                 tc_fence_before();
                 mbar_arrive(B(B_PF + (g & 1)));
@@ -593,20 +596,25 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             tc_fence_after();
             __syncwarp();
             const float ia = lta > 0.f ? 1.f / lta : 0.f, ib = ltb > 0.f ? 1.f / ltb : 0.f;
-            const uint32_t yslot = sb + kOffQ + 16384u * yb + 4u * (uint32_t)cq;
+            const uint32_t yrow = sb + kOffQ + 16384u * yb + (uint32_t)(16 * w + (lane & 7)) * 128u;
+            const uint32_t c0 = ((uint32_t)(lane >> 3) ^ (uint32_t)(lane & 7)) << 4;
+            const uint32_t c1 = ((uint32_t)((lane >> 3) + 4) ^ (uint32_t)(lane & 7)) << 4;
 #pragma unroll 1
             for (int h2 = 0; h2 < 2; ++h2) {
                 uint32_t yr[32];
                 tmem_ld16x256_x8(lbase + ycol + 64u * h2, yr);
                 tmem_wait_ld();
-                const uint32_t kb = yslot + 8192u * (uint32_t)h2;   // K-block of these 64 columns
+                uint32_t ya[8], yb8[8];
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
-                    st_shared_b32(kb + (uint32_t)ra * 128u + (((uint32_t)j ^ (uint32_t)(ra & 7)) << 4),
-                                  pack_bf16(__uint_as_float(yr[4 * j]) * ia, __uint_as_float(yr[4 * j + 1]) * ia));
-                    st_shared_b32(kb + (uint32_t)rb * 128u + (((uint32_t)j ^ (uint32_t)(rb & 7)) << 4),
-                                  pack_bf16(__uint_as_float(yr[4 * j + 2]) * ib, __uint_as_float(yr[4 * j + 3]) * ib));
+                    ya[j] = pack_bf16(__uint_as_float(yr[4 * j]) * ia, __uint_as_float(yr[4 * j + 1]) * ia);
+                    yb8[j] = pack_bf16(__uint_as_float(yr[4 * j + 2]) * ib, __uint_as_float(yr[4 * j + 3]) * ib);
                 }
+                const uint32_t kb = yrow + 8192u * (uint32_t)h2;   // K-block of these 64 columns
+                stmatrix_x4(kb + c0, ya[0], ya[1], ya[2], ya[3]);
+                stmatrix_x4(kb + c1, ya[4], ya[5], ya[6], ya[7]);
+                stmatrix_x4(kb + 1024u + c0, yb8[0], yb8[1], yb8[2], yb8[3]);
+                stmatrix_x4(kb + 1024u + c1, yb8[4], yb8[5], yb8[6], yb8[7]);
             }
             fence_async_smem();
             tc_fence_before();

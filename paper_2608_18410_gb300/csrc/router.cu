@@ -31,53 +31,261 @@ __global__ void k_lang_pool(const T *__restrict__ h, const rolesub_episode *__re
 }
 
 // beta[l][e][f] = b1[f] + alpha_lang * W1[f][d+C : 2d+C] . ctx[l][e]
-// A small GEMM per layer (episodes x F x d): 16 episodes x 64 outputs per
-// block, the hidden dimension streamed through shared memory in 64-wide
-// steps; every thread owns one episode and four outputs.
+// A small GEMM per layer (episodes x F x d) in fp32. A cluster of four
+// blocks shares one 64-episode x 32-output tile, each block a quarter of d;
+// every thread holds 4 episodes x 2 outputs. d runs in 64-wide steps through
+// shared memory, the next step's tiles loaded into registers meanwhile.
+// Ranks 1-3 then add into rank 0 through distributed shared memory, in rank
+// order, so the sum does not depend on timing.
+constexpr int kBiasSplit = 4;
+
+__device__ __forceinline__ uint32_t cluster_rank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ void cluster_sync()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 template <class T>
-__global__ void __launch_bounds__(256)
+__global__ void __cluster_dims__(kBiasSplit, 1, 1) __launch_bounds__(256)
 k_lang_bias(const T *__restrict__ W1, const float *__restrict__ b1, const float *__restrict__ ctx,
             int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
 {
-    constexpr int BE = 16, BF = 64, BK = 64, WP = BF + 4;   // WP: padded row pitch
-    __shared__ __align__(16) float Ws[BK * WP];             // [t][f]
-    __shared__ float Cs[BE][BK + 1];                        // [e][t]
-    const int l = blockIdx.z;
-    const int f0 = blockIdx.x * BF, e0 = blockIdx.y * BE;
-    const int te = threadIdx.x >> 4, tf = threadIdx.x & 15;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    constexpr int BE = 64, BF = 32, BK = 64, PE = BE + 4, PF = BF + 4;   // padded pitches
+    // Cs [t][e] and Ws [t][f]; afterwards the whole array holds the partial
+    // sums of ranks 1-3 (3 x 256 x 8 floats)
+    __shared__ __align__(16) float tiles[BK * PE + BK * PF];
+    static_assert(BK * PE + BK * PF >= (kBiasSplit - 1) * 256 * 8, "reduction buffer");
+    float(*Cs)[PE] = reinterpret_cast<float(*)[PE]>(tiles);
+    float(*Ws)[PF] = reinterpret_cast<float(*)[PF]>(tiles + BK * PE);
+    const int l = blockIdx.z, tid = threadIdx.x;
+    const uint32_t rank = cluster_rank();
+    const int f0 = (blockIdx.x / kBiasSplit) * BF, e0 = blockIdx.y * BE;
+    const int kper = ((d + kBiasSplit * BK - 1) / (kBiasSplit * BK)) * BK;
+    const int kb = (int)rank * kper, ke = min(d, kb + kper);
+    const int te = tid & 15, tf = tid >> 4;       // episodes e0 + 4te + i, outputs f0 + 2tf + j
     const size_t wstride = (size_t)(2 * d + C);
-    for (int k0 = 0; k0 < d; k0 += BK) {
-        for (int i = threadIdx.x; i < BF * BK; i += 256) {
-            const int ff = i / BK, t = i % BK;
-            const int f = f0 + ff;
-            Ws[t * WP + ff] = (f < F && k0 + t < d)
-                                   ? to_f(W1[((size_t)l * F + f) * wstride + d + C + k0 + t])
-                                   : 0.f;
+    const T *wbase = W1 + (size_t)l * F * wstride + d + C;
+    const float *cbase = ctx + (size_t)l * E * d;
+    // loaders, t fastest across a warp so that global reads are coalesced:
+    // ctx 64 episodes x 64 t (16 per thread), W 32 outputs x 64 t (8 per thread)
+    const int lt = tid & 63, lr = tid >> 6;
+    float cr[16], wr[8];
+    auto fetch = [&](int k0) {
+        const int t = k0 + lt;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const int e = e0 + lr + 4 * i;
+            cr[i] = (e < E && t < ke) ? cbase[(size_t)e * d + t] : 0.f;
         }
-        for (int i = threadIdx.x; i < BE * BK; i += 256) {
-            const int ee = i / BK, t = i % BK;
-            const int e = e0 + ee;
-            Cs[ee][t] = (e < E && k0 + t < d) ? ctx[((size_t)l * E + e) * d + k0 + t] : 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            const int f = f0 + lr + 4 * i;
+            wr[i] = (f < F && t < ke) ? to_f(wbase[(size_t)f * wstride + t]) : 0.f;
         }
+    };
+    float acc[8] = {};   // [i][j] = acc[2i + j]
+    if (kb < ke) fetch(kb);
+    for (int k0 = kb; k0 < ke; k0 += BK) {
+        __syncthreads();   // previous step's tiles are consumed
+#pragma unroll
+        for (int i = 0; i < 16; ++i) Cs[lt][lr + 4 * i] = cr[i];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) Ws[lt][lr + 4 * i] = wr[i];
         __syncthreads();
+        if (k0 + BK < ke) fetch(k0 + BK);
 #pragma unroll 16
         for (int t = 0; t < BK; ++t) {
-            const float c = Cs[te][t];
-            const float4 w = *reinterpret_cast<const float4 *>(&Ws[t * WP + 4 * tf]);
-            acc[0] = fmaf(c, w.x, acc[0]);
-            acc[1] = fmaf(c, w.y, acc[1]);
-            acc[2] = fmaf(c, w.z, acc[2]);
-            acc[3] = fmaf(c, w.w, acc[3]);
+            const float4 c = *reinterpret_cast<const float4 *>(&Cs[t][4 * te]);
+            const float2 w = *reinterpret_cast<const float2 *>(&Ws[t][2 * tf]);
+            acc[0] = fmaf(c.x, w.x, acc[0]);
+            acc[1] = fmaf(c.x, w.y, acc[1]);
+            acc[2] = fmaf(c.y, w.x, acc[2]);
+            acc[3] = fmaf(c.y, w.y, acc[3]);
+            acc[4] = fmaf(c.z, w.x, acc[4]);
+            acc[5] = fmaf(c.z, w.y, acc[5]);
+            acc[6] = fmaf(c.w, w.x, acc[6]);
+            acc[7] = fmaf(c.w, w.y, acc[7]);
+        }
+    }
+    // every block is done with its tiles; ranks 1-3 write their partial sums
+    // into rank 0's tile array, thread-major
+    __syncthreads();
+    cluster_sync();
+    if (rank != 0) {
+        const uint32_t local = static_cast<uint32_t>(__cvta_generic_to_shared(tiles)) +
+                               4u * (((rank - 1) * 256u + (uint32_t)tid) * 8u);
+        uint32_t remote;
+        asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(0u));
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote + 4u * q), "f"(acc[q]) : "memory");
+    }
+    cluster_sync();
+    if (rank != 0) return;
+    const float *red = tiles;
+#pragma unroll
+    for (int r = 0; r < kBiasSplit - 1; ++r)
+#pragma unroll
+        for (int q = 0; q < 8; ++q) acc[q] += red[(r * 256 + tid) * 8 + q];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int e = e0 + 4 * te + i;
+        if (e >= E) continue;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const int f = f0 + 2 * tf + j;
+            if (f < F) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * acc[2 * i + j];
+        }
+    }
+}
+
+// bf16 weights: the same product on the tensor cores (mma.sync m16n8k16,
+// fp32 accumulation). ctx is split into bf16 parts hi + lo (together exact to
+// about 2^-16 relative) and both are multiplied by the bf16 weights. Block:
+// 64 episodes x 64 outputs x half of d, four warps of 16 episodes each; a
+// cluster of two blocks along d adds rank 1 into rank 0 through distributed
+// shared memory. Needs d % 128 == 0 and C % 8 == 0 (16-byte weight rows).
+constexpr int kMmaSplit = 2;
+
+__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
+                 : "r"(addr));
+}
+
+__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                          uint32_t b0, uint32_t b1)
+{
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+                 "{%8, %9}, {%0, %1, %2, %3};"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ uint32_t pack2(float a, float b)
+{
+    const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<const uint32_t *>(&v);
+}
+
+__global__ void __cluster_dims__(kMmaSplit, 1, 1) __launch_bounds__(128)
+k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *__restrict__ ctx,
+                int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
+{
+    constexpr int BE = 64, BF = 64, BK = 64;
+    // rows of 64 bf16 (128 B) as 8 16-byte chunks, chunk c of row r stored at
+    // position c ^ (r % 8) so that ldmatrix rows hit distinct banks
+    __shared__ __align__(128) uint8_t sm[3 * BE * BK * 2];   // A hi, A lo, B; later rank 1's sums
+    const uint32_t sA0 = static_cast<uint32_t>(__cvta_generic_to_shared(sm));
+    const uint32_t sA1 = sA0 + BE * BK * 2, sBs = sA1 + BE * BK * 2;
+    const int l = blockIdx.z, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t rank = cluster_rank();
+    const int f0 = (blockIdx.x / kMmaSplit) * BF, e0 = blockIdx.y * BE;
+    const int kper = d / kMmaSplit;
+    const int kb = (int)rank * kper, ke = kb + kper;
+    const size_t wstride = (size_t)(2 * d + C);
+    const __nv_bfloat16 *wbase = W1 + (size_t)l * F * wstride + d + C;
+    const float *cbase = ctx + (size_t)l * E * d;
+    float4 cr[8];
+    uint4 wr[4];
+    auto fetch = [&](int k0) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {   // ctx: row e, float4 kq of the 64-wide step
+            const int idx = tid + 128 * j, e = e0 + (idx >> 4), kq = idx & 15;
+            cr[j] = e < E ? *reinterpret_cast<const float4 *>(cbase + (size_t)e * d + k0 + 4 * kq)
+                          : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {   // W: row f, 16-byte chunk c
+            const int idx = tid + 128 * j, f = f0 + (idx >> 3), c = idx & 7;
+            wr[j] = f < F ? *reinterpret_cast<const uint4 *>(wbase + (size_t)f * wstride + k0 + 8 * c)
+                          : make_uint4(0, 0, 0, 0);
+        }
+    };
+    float acc[8][4] = {};
+    fetch(kb);
+    for (int k0 = kb; k0 < ke; k0 += BK) {
+        __syncthreads();   // previous step's tiles are consumed
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            const int idx = tid + 128 * j, e = idx >> 4, kq = idx & 15;
+            const float4 v = cr[j];
+            const uint32_t h0 = pack2(v.x, v.y), h1 = pack2(v.z, v.w);
+            const __nv_bfloat162 hb0 = *reinterpret_cast<const __nv_bfloat162 *>(&h0);
+            const __nv_bfloat162 hb1 = *reinterpret_cast<const __nv_bfloat162 *>(&h1);
+            const uint32_t l0 = pack2(v.x - __low2float(hb0), v.y - __high2float(hb0));
+            const uint32_t l1 = pack2(v.z - __low2float(hb1), v.w - __high2float(hb1));
+            const uint32_t off = (uint32_t)e * 128u + ((((uint32_t)kq >> 1) ^ ((uint32_t)e & 7u)) << 4) +
+                                 ((uint32_t)kq & 1u) * 8u;
+            asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(sA0 + off), "r"(h0), "r"(h1) : "memory");
+            asm volatile("st.shared.v2.b32 [%0], {%1, %2};" ::"r"(sA1 + off), "r"(l0), "r"(l1) : "memory");
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int idx = tid + 128 * j, f = idx >> 3, c = idx & 7;
+            const uint32_t off = (uint32_t)f * 128u + (((uint32_t)c ^ ((uint32_t)f & 7u)) << 4);
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(sBs + off), "r"(wr[j].x), "r"(wr[j].y),
+                         "r"(wr[j].z), "r"(wr[j].w)
+                         : "memory");
         }
         __syncthreads();
-    }
-    const int e = e0 + te;
-    if (e >= E) return;
+        if (k0 + BK < ke) fetch(k0 + BK);
 #pragma unroll
-    for (int j = 0; j < 4; ++j) {
-        const int f = f0 + 4 * tf + j;
-        if (f < F) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * acc[j];
+        for (int s16 = 0; s16 < BK / 16; ++s16) {
+            const uint32_t ar = (uint32_t)(16 * warp + (lane & 15));
+            const uint32_t aoff = ar * 128u + ((((uint32_t)(2 * s16 + (lane >> 4))) ^ (ar & 7u)) << 4);
+            uint32_t ah[4], al[4];
+            ldsm_x4(sA0 + aoff, ah[0], ah[1], ah[2], ah[3]);
+            ldsm_x4(sA1 + aoff, al[0], al[1], al[2], al[3]);
+#pragma unroll
+            for (int pr = 0; pr < 4; ++pr) {   // output tiles 2pr, 2pr + 1
+                const uint32_t n = (uint32_t)(16 * pr + (lane & 7) + ((lane >> 4) << 3));
+                const uint32_t boff = n * 128u + ((((uint32_t)(2 * s16 + ((lane >> 3) & 1))) ^ (n & 7u)) << 4);
+                uint32_t b0, b1, b2, b3;
+                ldsm_x4(sBs + boff, b0, b1, b2, b3);
+                mma_16816(acc[2 * pr], ah[0], ah[1], ah[2], ah[3], b0, b1);
+                mma_16816(acc[2 * pr], al[0], al[1], al[2], al[3], b0, b1);
+                mma_16816(acc[2 * pr + 1], ah[0], ah[1], ah[2], ah[3], b2, b3);
+                mma_16816(acc[2 * pr + 1], al[0], al[1], al[2], al[3], b2, b3);
+            }
+        }
+    }
+    // rank 1 adds its sums into rank 0 (thread-major, 128 x 32 floats)
+    __syncthreads();
+    cluster_sync();
+    if (rank != 0) {
+        const uint32_t local = sA0 + 4u * ((uint32_t)tid * 32u);
+        uint32_t remote;
+        asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(0u));
+#pragma unroll
+        for (int q = 0; q < 32; ++q)
+            asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote + 4u * q), "f"(acc[q >> 2][q & 3]) : "memory");
+    }
+    cluster_sync();
+    if (rank != 0) return;
+    const float *red = reinterpret_cast<const float *>(sm) + tid * 32;
+#pragma unroll
+    for (int q = 0; q < 32; ++q) acc[q >> 2][q & 3] += red[q];
+    const int g = lane >> 2, t2 = 2 * (lane & 3);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const int e = e0 + 16 * warp + g + 8 * h;
+            if (e >= E) continue;
+#pragma unroll
+            for (int q = 0; q < 2; ++q) {
+                const int f = f0 + 8 * j + t2 + q;
+                if (f < F) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * acc[j][2 * h + q];
+            }
+        }
     }
 }
 
@@ -231,8 +439,12 @@ static cudaError_t launch_router_t(const CompressArgs &a)
             *W2 = (const T *)a.W2;
     k_lang_pool<T><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
         h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
-    k_lang_bias<T><<<dim3((F + 63) / 64, (E + 15) / 16, L), 256, 0, a.stream>>>(
-        W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+    if (sizeof(T) == 2 && d % 128 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
+        k_lang_bias_mma<<<dim3((F + 63) / 64 * kMmaSplit, (E + 63) / 64, L), 128, 0, a.stream>>>(
+            (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+    else
+        k_lang_bias<T><<<dim3((F + 31) / 32 * kBiasSplit, (E + 63) / 64, L), 256, 0, a.stream>>>(
+            W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
     if (router_tc_supported(a.shape)) {
         count_launches(2);
         cudaError_t e = cudaGetLastError();

@@ -65,10 +65,32 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
     return ok != 0;
 }
 
-// Polls until the phase with the given parity has completed. Gives up after
-// a bounded number of polls (seconds), or at once when *abort is set by a
-// thread that already gave up; returns false in both cases.
-constexpr uint32_t kMaxPolls = 1u << 24;
+// try_wait with a suspend-time hint: the thread sleeps until the phase
+// completes or about `ns` nanoseconds pass, instead of spinning.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t ns)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+        " selp.b32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(ns)
+        : "memory");
+    return ok != 0;
+}
+
+__device__ __forceinline__ uint64_t global_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+    return t;
+}
+
+// Waits until the phase with the given parity has completed. Gives up after
+// about two seconds, or soon after *abort is set by a thread that already
+// gave up; returns false in both cases.
+constexpr uint64_t kWaitLimitNs = 2000000000ull;
+constexpr uint32_t kSleepHintNs = 100000;
 
 // Cold path of a wait that ran out: records where and tells the other roles.
 // Kept out of line so that every inlined wait stays a few instructions long.
@@ -81,10 +103,13 @@ static __device__ __noinline__ void wait_timed_out(int32_t *status, volatile int
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status,
                                           volatile int *abort, int where)
 {
+    if (mbar_try_wait_sleep(bar, parity, kSleepHintNs)) return true;
+    const uint64_t t0 = global_ns();
 #pragma unroll 1
-    for (uint32_t i = 0; i < kMaxPolls; ++i) {
-        if (mbar_try_wait(bar, parity)) return true;
-        if ((i & 255u) == 255u && *abort) return false;
+    for (;;) {
+        if (mbar_try_wait_sleep(bar, parity, kSleepHintNs)) return true;
+        if (*abort) return false;
+        if (global_ns() - t0 > kWaitLimitNs) break;
     }
     wait_timed_out(status, abort, where);
     return false;
@@ -254,6 +279,16 @@ __device__ __forceinline__ void tmem_st16x256_x1(uint32_t taddr, const uint32_t 
 {
     asm volatile("tcgen05.st.sync.aligned.16x256b.x1.b32 [%0], {%1, %2, %3, %4};" ::"r"(taddr), "r"(r[0]),
                  "r"(r[1]), "r"(r[2]), "r"(r[3])
+                 : "memory");
+}
+
+// Four 8x8 b16 matrices, each in the fragment layout where thread t holds
+// row t/4, columns 2(t%4) + {0, 1} (one 32-bit register per matrix), to
+// shared memory; lane t supplies the address of row t%8 of matrix t/8.
+__device__ __forceinline__ void stmatrix_x4(uint32_t addr, uint32_t r0, uint32_t r1, uint32_t r2, uint32_t r3)
+{
+    asm volatile("stmatrix.sync.aligned.m8n8.x4.shared.b16 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(r0), "r"(r1),
+                 "r"(r2), "r"(r3)
                  : "memory");
 }
 
