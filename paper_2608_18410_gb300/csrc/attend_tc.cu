@@ -27,27 +27,30 @@
 //         to its slot; per-row records (kept ids, packed offset) are fetched
 //         three chunks ahead.
 //   Y += P_c Z_c                   tcgen05, M=64, N=128 (rotated space)
-// Unit tail: Y / l -> bf16 smem (into the unit's finished Q slot),
+// Unit tail: Y / l -> bf16 smem (a staging tile of its own, so that a Q
+// slot is free as soon as its unit's last S is issued),
 // O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into the unit's Y buffer, output
 // stores.
 //
-// Warp roles (384 threads), all hand-offs through mbarriers:
+// Warp roles (512 threads), all hand-offs through mbarriers. Warp w runs on
+// sub-partition w % 4.
 //   warps 0-3   softmax, one per TMEM lane quadrant
-//   warps 4,5   value gather, one kv row per thread
-//   warp 6      TMA producer: K (4-slot ring), Q (2 slots), R_h
-//   warp 7      MMA issuer: a non-blocking loop over three cursors (next S,
-//               next P.Z, next output product) that issues whichever is
-//               ready, in order within each cursor
+//   warps 4-5, 12-13  value gather, one kv row per thread: warps 4-5 the
+//               even chunks, warps 12-13 the odd ones
+//   warp 6      issues S = Q K^T, chunk by chunk
+//   warp 14     issues Y += P Z, chunk by chunk
+//   warp 15     issues O = Y R_h^T, unit by unit
+//   warp 7      TMA producer: K (3-slot ring), Q (2 slots), R_h
 //   warps 8-11  unit tail, one per lane quadrant, overlapping the next
 //               unit's chunks (Y is double buffered in TMEM)
 // P is double buffered and Z has four slots: a chunk's softmax waits for the
-// product two chunks back, its gather for the one four chunks back, and the
-// gather publishes a chunk two iterations after issuing its copies.
+// product two chunks back, its gatherer for the one four chunks back, and a
+// gatherer publishes a chunk when it starts its next one.
 //
 // Shared memory (1024-aligned):
-//   0K   Q[2]   16K each (two 64-column K-blocks of 64 rows); the unit tail
-//                writes Y / l into its own Q slot
-//   32K  K[4]   16K each (64-row chunks)
+//   0K   Q[2]   16K each (two 64-column K-blocks of 64 rows)
+//   32K  K[3]   16K each (64-row chunks)
+//   80K  Y      16K, Y / l of the unit in its tail (A of the output product)
 //   96K  R_h    32K (two 64-column K-blocks of 128 rows)
 //   128K P[2]   8K each (64 rows x 64 kv)
 //   144K Z[4]   16K each (two 64-column MN-blocks of 64 kv rows)
@@ -71,17 +74,18 @@ namespace {
 using namespace sm100;
 typedef __nv_bfloat16 bf16;
 
-constexpr int kThreads = 384;
+constexpr int kThreads = 512;
 constexpr int kChunk = 64;   // cache tokens per chunk
 constexpr int kQRows = 64;   // query rows per unit
 constexpr int kDh = 128;
 constexpr int kG = 16;       // groups per head (d_s = 8)
 constexpr int kMaxUnits = 448;   // units per CTA and launch (unit list in smem)
-constexpr int kKSlots = 4;
+constexpr int kKSlots = 3;
 constexpr float kRescaleLog2 = 8.f;   // raise the reference max beyond 2^8 growth
 
 constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = 32768;
+constexpr uint32_t kOffY = kOffK + kKSlots * 16384;   // normalised Y of the unit in its tail
 constexpr uint32_t kOffR = 98304;
 constexpr uint32_t kOffP = 131072;
 constexpr uint32_t kOffZ = 147456;                   // 4 x 16K ring
@@ -256,7 +260,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
     tc_fence_after();
     const uint32_t tmem = tmem_slot;
 
-    if (warp == 6) {
+    if (warp == 7) {
         // ================= TMA producer =================================
         if (lane == 0) {
             prefetch_tmap(&tm_q);
@@ -304,116 +308,120 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 ++n;
             }
         }
-    } else if (warp == 7) {
-        // ================= MMA issuer (non-blocking over three cursors) ====
-        // tcgen05.mma issue stalls while the tensor pipe is busy, so the work
-        // between products is kept minimal: every shared-memory descriptor is
-        // a base computed here plus a constant (offset / 16 in the start
-        // address field, which cannot carry out of its 14 bits below 256 KB).
-        if (lane == 0) {
+    } else if (warp == 6 || warp == 14 || warp == 15) {
+        // ================= MMA issuers =====================================
+        // Three threads in three warps, one per product, each walking its
+        // chunks or units in order with blocking waits; the tensor pipe
+        // interleaves what they issue. tcgen05.mma issue stalls while the
+        // pipe is busy, so the work between products is kept minimal: every
+        // shared-memory descriptor is a base plus a constant (offset / 16 in
+        // the start address field, which cannot carry out of its 14 bits
+        // below 256 KB). A commit tracks the issuing thread's own products.
+        if (lane == 0 && warp == 6) {
+            // S_g = Q K_g^T into S buffer g % 2
             const uint64_t dq = sdesc_sw128(sb + kOffQ, 16, 1024), dk = sdesc_sw128(sb + kOffK, 16, 1024);
+            ChunkIt cs = first;
+            uint32_t gs = 0, ns = 0;   // chunk counter, unit counter
+            while (cs.k < nu) {
+                const uint32_t ks = gs % kKSlots;
+                // S buffer gs % 2 was read by the softmax of chunk gs - 2
+                if (gs >= 2 && !mbar_wait(B(B_PF + (gs & 1)), ((gs - 2) >> 1) & 1, status, &abort_flag, 50)) break;
+                if (cs.c == 0 && !mbar_wait(B(B_QF + (ns & 1)), (ns >> 1) & 1, status, &abort_flag, 51)) break;
+                if (!mbar_wait(B(B_KF + ks), (gs / kKSlots) & 1, status, &abort_flag, 52)) break;
+                tc_fence_after();
+                const uint64_t qd = dq + 1024u * (ns & 1), kd = dk + 1024u * ks;
+                const uint32_t sc = tmem + kColS + 64u * (gs & 1);
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint32_t o16 = (kk >> 2) * 512u + (kk & 3) * 2u;   // (kk/4) * 8K + (kk%4) * 32 bytes
+                    mma_bf16(sc, qd + o16, kd + o16, kIdescS, kk > 0);
+                }
+                mma_commit(B(B_SF + (gs & 1)));
+                mma_commit(B(B_KE + ks));
+                if (it_next(sp, cs, nu)) {
+                    mma_commit(B(B_QE + (ns & 1)));   // the unit's last S: its Q slot is free
+                    ++ns;
+                }
+                ++gs;
+            }
+        } else if (lane == 0 && warp == 14) {
+            // Y += P_g Z_g; a unit's first product starts its Y buffer afresh,
+            // once the unit two back has had its output read from it
             const uint64_t dp = sdesc_sw128(sb + kOffP, 16, 1024), dz = sdesc_sw128(sb + kOffZ, 8192, 1024);
-            const uint64_t dr = sdesc_sw128(sb + kOffR, 16, 1024);
-            ChunkIt cs = first, cp = first, co = first;
-            uint32_t gs = 0, ns = 0;   // next S: chunk counter, unit counter
-            uint32_t gp = 0, np = 0;   // next P.Z
-            uint32_t no = 0;           // next output product (unit counter)
+            ChunkIt cp = first;
+            uint32_t gp = 0, np = 0;
+            while (cp.k < nu) {
+                const uint32_t yb = np & 1, b = gp & 1, zs = gp & 3;
+                if (cp.c == 0 && np >= 2 && !mbar_wait(B(B_OE + yb), ((np - 2) >> 1) & 1, status, &abort_flag, 53))
+                    break;
+                if (!mbar_wait(B(B_PF + b), (gp >> 1) & 1, status, &abort_flag, 54)) break;
+                if (!mbar_wait(B(B_ZF + zs), (gp >> 2) & 1, status, &abort_flag, 55)) break;
+                tc_fence_after();
+                const uint64_t pd = dp + 512u * b, zd = dz + 1024u * zs;
+                const uint32_t yc = tmem + kColY + 128u * yb;
+                mma_bf16(yc, pd, zd, kIdescPV, cp.c > 0 ? 1u : 0u);
+#pragma unroll
+                for (int kk = 1; kk < 4; ++kk)   // P: +32 bytes, Z: +16 kv rows (2 KB) per step
+                    mma_bf16(yc, pd + 2u * kk, zd + 128u * kk, kIdescPV, 1u);
+                mma_commit(B(B_PV + zs));
+                if (it_next(sp, cp, nu)) {
+                    mma_commit(B(B_YR + yb));   // the unit's Y is complete
+                    ++np;
+                }
+                ++gp;
+            }
+        } else if (lane == 0) {
+            // O = Y R_h^T of each unit, from its normalised Y in shared memory,
+            // written over that unit's Y buffer
+            const uint64_t dr = sdesc_sw128(sb + kOffR, 16, 1024), yd = sdesc_sw128(sb + kOffY, 16, 1024);
+            ChunkIt co = first;
+            uint32_t no = 0;
             int run_o = 0;
-            uint32_t idle = 0;
-            while (co.k < nu && !abort_flag) {
-                bool prog = false;
-                // S of the next chunk: its S buffer is free once P.Z two chunks back
-                // has been issued (that needed the softmax to have read it)
-                if (cs.k < nu && gs <= gp + 1) {
-                    const uint32_t ks = gs % kKSlots;
-                    const bool qok = cs.c > 0 || mbar_test(B(B_QF + (ns & 1)), (ns >> 1) & 1);
-                    if (qok && mbar_test(B(B_KF + ks), (gs / kKSlots) & 1)) {
-                        tc_fence_after();
-                        const uint64_t qd = dq + 1024u * (ns & 1), kd = dk + 1024u * ks;
-                        const uint32_t sc = tmem + kColS + 64u * (gs & 1);
+            while (co.k < nu) {
+                if (!mbar_wait(B(B_YF), no & 1, status, &abort_flag, 56)) break;
+                if (!mbar_wait(B(B_RF), run_o & 1, status, &abort_flag, 57)) break;
+                tc_fence_after();
+                const uint32_t oc = tmem + kColY + 128u * (no & 1);
 #pragma unroll
-                        for (int kk = 0; kk < 8; ++kk) {
-                            const uint32_t o16 = (kk >> 2) * 512u + (kk & 3) * 2u;   // (kk/4) * 8K + (kk%4) * 32 bytes
-                            mma_bf16(sc, qd + o16, kd + o16, kIdescS, kk > 0);
-                        }
-                        mma_commit(B(B_SF + (gs & 1)));
-                        mma_commit(B(B_KE + ks));
-                        if (it_next(sp, cs, nu)) ++ns;
-                        ++gs;
-                        prog = true;
-                    }
+                for (int kk = 0; kk < 8; ++kk) {
+                    const uint32_t a16 = (kk >> 2) * 512u + (kk & 3) * 2u;    // Y: 8K K-blocks
+                    const uint32_t b16 = (kk >> 2) * 1024u + (kk & 3) * 2u;   // R_h: 16K K-blocks
+                    mma_bf16(oc, yd + a16, dr + b16, kIdescO, kk > 0);
                 }
-                // P.Z of the next chunk; a unit's first one starts its Y buffer
-                // afresh, once the unit two back has had its output read from it
-                if (cp.k < nu) {
-                    const uint32_t yb = np & 1, b = gp & 1, zs = gp & 3;
-                    const bool yfree = cp.c > 0 || np < 2 || mbar_test(B(B_OE + yb), ((np - 2) >> 1) & 1);
-                    if (yfree && mbar_test(B(B_PF + b), (gp >> 1) & 1) && mbar_test(B(B_ZF + zs), (gp >> 2) & 1)) {
-                        tc_fence_after();
-                        const uint64_t pd = dp + 512u * b, zd = dz + 1024u * zs;
-                        const uint32_t yc = tmem + kColY + 128u * yb;
-                        mma_bf16(yc, pd, zd, kIdescPV, cp.c > 0 ? 1u : 0u);
-#pragma unroll
-                        for (int kk = 1; kk < 4; ++kk)   // P: +32 bytes, Z: +16 kv rows (2 KB) per step
-                            mma_bf16(yc, pd + 2u * kk, zd + 128u * kk, kIdescPV, 1u);
-                        mma_commit(B(B_PV + zs));
-                        if (it_next(sp, cp, nu)) {
-                            mma_commit(B(B_YR + yb));   // the unit's Y is complete
-                            ++np;
-                        }
-                        ++gp;
-                        prog = true;
-                    }
+                mma_commit(B(B_OF));
+                ChunkIt nx = co;
+                next_unit(sp, nx, nu);
+                if (nx.k >= nu || nx.t.l != co.t.l || nx.t.h != co.t.h) {
+                    mma_commit(B(B_RE));
+                    ++run_o;
                 }
-                // output product O = Y R_h^T of the oldest unit whose normalised Y is
-                // in shared memory; written over that unit's Y buffer
-                if (np > no) {
-                    if (mbar_test(B(B_YF), no & 1) && mbar_test(B(B_RF), run_o & 1)) {
-                        tc_fence_after();
-                        const uint64_t yd = dq + 1024u * (no & 1);
-                        const uint32_t oc = tmem + kColY + 128u * (no & 1);
-#pragma unroll
-                        for (int kk = 0; kk < 8; ++kk) {
-                            const uint32_t a16 = (kk >> 2) * 512u + (kk & 3) * 2u;    // Y: 8K K-blocks
-                            const uint32_t b16 = (kk >> 2) * 1024u + (kk & 3) * 2u;   // R_h: 16K K-blocks
-                            mma_bf16(oc, yd + a16, dr + b16, kIdescO, kk > 0);
-                        }
-                        mma_commit(B(B_OF));
-                        mma_commit(B(B_QE + (no & 1)));   // Q slot (and the Y in it) free
-                        ChunkIt nx = co;
-                        next_unit(sp, nx, nu);
-                        if (nx.k >= nu || nx.t.l != co.t.l || nx.t.h != co.t.h) {
-                            mma_commit(B(B_RE));
-                            ++run_o;
-                        }
-                        co = nx;
-                        ++no;
-                        prog = true;
-                    }
-                }
-                if (prog) {
-                    idle = 0;
-                } else if (++idle > (1u << 26)) {
-                    report(status, ROLESUB_ETIMEOUT, 59);
-                    abort_flag = 1;
-                }
+                co = nx;
+                ++no;
             }
         }
-    } else if (warp == 4 || warp == 5) {
+    } else if (warp == 4 || warp == 5 || warp == 12 || warp == 13) {
         // ================= value gather (one kv row per thread) ===========
-        // Chunk g goes to Z slot g % 4. Its row record is fetched three chunks
-        // ahead; at iteration g the kept groups of chunk g are copied by
-        // cp.async straight into their swizzled slots of the tile, groups
-        // left over from the slot's previous chunk are zeroed, and the copies
-        // of chunk g - 2 (two commit groups back) are published to the MMA
-        // warp.
-        const int jl = tid - 128;
+        // Two gatherers of 64 threads (warps 4-5 and 12-13) take the even and
+        // the odd chunks. Chunk g goes to Z slot g % 4; its row record is
+        // fetched one own chunk (two chunks) ahead. At chunk g a gatherer
+        // publishes its previous chunk g - 2 (copies complete), waits for
+        // the product of chunk g - 4 to free the slot, copies the kept
+        // groups of chunk g by cp.async straight into their swizzled slots of
+        // the tile and zeroes the groups left over from the slot's previous
+        // chunk.
+        const int par = warp >= 12 ? 1 : 0, jl = tid & 63;   // warps 12-13: odd chunks
         const uint32_t sw = (uint32_t)(jl & 7);
         // groups of this thread's row that may be non-zero, per Z slot (16 bits
         // each); a slot's first use clears everything
         uint64_t dirty = ~0ull;
-        ChunkIt ahead = first, it = first;
-        auto stage_rec = [&](uint32_t gg) {
+        ChunkIt it = first;
+        uint32_t g = 0;
+        if (par == 1) {
+            it_next(sp, it, nu);
+            g = 1;
+        }
+        ChunkIt ahead = it;
+        auto stage_rec = [&](uint32_t gg) {   // record of chunk gg (= ahead), then ahead += 2
             if (ahead.k < nu) {
                 const int r = ahead.c * kChunk + jl;
                 if (r < ahead.t.nc)
@@ -421,14 +429,12 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                                rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
             }
             it_next(sp, ahead, nu);
+            it_next(sp, ahead, nu);
             cp_async_commit();
         };
-        stage_rec(0);
-        stage_rec(1);
-        stage_rec(2);
-        uint32_t g = 0;
-        for (; it.k < nu && !abort_flag; ++g) {
-            cp_async_wait_group<1>();   // record g and the copies of chunk g - 2 have landed
+        stage_rec(g);
+        for (; it.k < nu && !abort_flag; g += 2) {
+            cp_async_wait_group<0>();   // record g and the copies of chunk g - 2 have landed
             if (g >= 2) {
                 fence_async_smem();
                 mbar_arrive(B(B_ZF + ((g - 2) & 3u)));
@@ -456,13 +462,13 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 st_shared_v4(zrow + (gg >> 3) * 8192u + (((gg & 7u) ^ sw) << 4), 0, 0, 0, 0);
             }
             dirty = (dirty & ~(0xFFFFull << sh)) | ((uint64_t)kept << sh);
-            stage_rec(g + 3);   // also commits this chunk's copies
+            stage_rec(g + 2);   // also commits this chunk's copies
+            it_next(sp, it, nu);
             it_next(sp, it, nu);
         }
         cp_async_wait_group<0>();
         fence_async_smem();
-        if (g >= 2) mbar_arrive(B(B_ZF + ((g - 2) & 3u)));
-        if (g >= 1) mbar_arrive(B(B_ZF + ((g - 1) & 3u)));
+        if (g >= 2 + (uint32_t)par) mbar_arrive(B(B_ZF + ((g - 2) & 3u)));
     } else if (warp < 4) {
         // ================= softmax (warps 0-3) ============================
         // rows ra = 16w + lane/4 and rb = ra + 8 of the unit; column pairs
@@ -577,7 +583,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             next_unit(sp, it, nu);
             ++n;
         }
-    } else {
+    } else if (warp >= 8 && warp < 12) {
         // ================= unit tail (warps 8-11) =========================
         // y / l -> bf16 operand in the unit's Q slot; after O = Y R_h^T, the
         // output rows. Lane quadrant w = warp % 4, same row mapping as softmax.
@@ -596,7 +602,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             tc_fence_after();
             __syncwarp();
             const float ia = lta > 0.f ? 1.f / lta : 0.f, ib = ltb > 0.f ? 1.f / ltb : 0.f;
-            const uint32_t yrow = sb + kOffQ + 16384u * yb + (uint32_t)(16 * w + (lane & 7)) * 128u;
+            const uint32_t yrow = sb + kOffY + (uint32_t)(16 * w + (lane & 7)) * 128u;
             const uint32_t c0 = ((uint32_t)(lane >> 3) ^ (uint32_t)(lane & 7)) << 4;
             const uint32_t c1 = ((uint32_t)((lane >> 3) + 4) ^ (uint32_t)(lane & 7)) << 4;
 #pragma unroll 1
