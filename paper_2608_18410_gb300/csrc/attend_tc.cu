@@ -29,7 +29,7 @@
 //   Y += P_c Z_c                   tcgen05, M=64, N=128 (rotated space)
 // Unit tail: Y / l -> bf16 smem (a staging tile of its own, so that a Q
 // slot is free as soon as its unit's last S is issued),
-// O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into the unit's Y buffer, output
+// O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into its own accumulator, output
 // stores.
 //
 // Warp roles (512 threads), all hand-offs through mbarriers. Warp w runs on
@@ -57,8 +57,7 @@
 //   208K records 4 x 1K
 //   212K row sums 2 x 64 fp32 (softmax -> unit tail)
 //   then the episode table and the barriers
-// TMEM (384 of 512 columns): S[2] at 0 and 64, Y[2] at 128 and 256 (each
-// later holding its unit's O).
+// TMEM (512 columns): S[2] at 0 and 64, Y[2] at 128 and 256, O at 384.
 #include <cuda.h>
 
 #include <algorithm>
@@ -96,7 +95,7 @@ constexpr uint32_t kOffUnits = kOffL + 1024;         // kMaxUnits x 16 B unit re
 constexpr uint32_t kOffBar = kOffUnits + 16 * kMaxUnits;
 constexpr uint32_t kSmemBytes = kOffBar + 512 + 1024;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0, kColY = 128;   // Y[b] at kColY + 128b
+constexpr uint32_t kColS = 0, kColY = 128, kColO = 384;   // Y[b] at kColY + 128b
 
 constexpr uint32_t kIdescS = idesc_bf16(64, 64, false);
 constexpr uint32_t kIdescPV = idesc_bf16(64, 128, true);
@@ -105,7 +104,7 @@ constexpr uint32_t kIdescO = idesc_bf16(64, 128, false);
 // barrier slots (8 bytes each); [2] / [4] entries are per buffer
 enum {
     B_QF = 0, B_QE = 2, B_KF = 4, B_KE = 8, B_RF = 12, B_RE = 13, B_SF = 14, B_PF = 16, B_ZF = 18, B_PV = 22,
-    B_YR = 26, B_YF = 28, B_OF = 29, B_OE = 30, B_LF = 32, B_COUNT = 34
+    B_YR = 26, B_YF = 28, B_OF = 30, B_OE = 31, B_LF = 32, B_COUNT = 34
 };
 
 struct Unit {
@@ -197,7 +196,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         abort_flag = 0;
         for (int i = 0; i < B_COUNT; ++i) {
             uint32_t cnt = 1;
-            if (i == B_PF || i == B_PF + 1 || i == B_YF || i == B_OE || i == B_OE + 1 || i == B_LF || i == B_LF + 1)
+            if (i == B_PF || i == B_PF + 1 || i == B_YF || i == B_YF + 1 || i == B_OE || i == B_LF || i == B_LF + 1)
                 cnt = 128;
             if (i >= B_ZF && i < B_ZF + kZSlots) cnt = 64;
             mbar_init(B(i), cnt);
@@ -346,13 +345,13 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             }
         } else if (lane == 0 && warp == 14) {
             // Y += P_g Z_g; a unit's first product starts its Y buffer afresh,
-            // once the unit two back has had its output read from it
+            // once the tail of the unit two back has read it
             const uint64_t dp = sdesc_sw128(sb + kOffP, 16, 1024), dz = sdesc_sw128(sb + kOffZ, 8192, 1024);
             ChunkIt cp = first;
             uint32_t gp = 0, np = 0;
             while (cp.k < nu) {
                 const uint32_t yb = np & 1, b = gp & 1, zs = gp & 3;
-                if (cp.c == 0 && np >= 2 && !mbar_wait(B(B_OE + yb), ((np - 2) >> 1) & 1, status, &abort_flag, 53))
+                if (cp.c == 0 && np >= 2 && !mbar_wait(B(B_YF + yb), ((np - 2) >> 1) & 1, status, &abort_flag, 53))
                     break;
                 if (!mbar_wait(B(B_PF + b), (gp >> 1) & 1, status, &abort_flag, 54)) break;
                 if (!mbar_wait(B(B_ZF + zs), (gp >> 2) & 1, status, &abort_flag, 55)) break;
@@ -371,17 +370,18 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 ++gp;
             }
         } else if (lane == 0) {
-            // O = Y R_h^T of each unit, from its normalised Y in shared memory,
-            // written over that unit's Y buffer
+            // O = Y R_h^T of each unit, from its normalised Y in shared memory
             const uint64_t dr = sdesc_sw128(sb + kOffR, 16, 1024), yd = sdesc_sw128(sb + kOffY, 16, 1024);
             ChunkIt co = first;
             uint32_t no = 0;
             int run_o = 0;
             while (co.k < nu) {
-                if (!mbar_wait(B(B_YF), no & 1, status, &abort_flag, 56)) break;
+                if (!mbar_wait(B(B_YF + (no & 1)), (no >> 1) & 1, status, &abort_flag, 56)) break;
+                // the O accumulator was read by the tail of the previous unit
+                if (no >= 1 && !mbar_wait(B(B_OE), (no - 1) & 1, status, &abort_flag, 58)) break;
                 if (!mbar_wait(B(B_RF), run_o & 1, status, &abort_flag, 57)) break;
                 tc_fence_after();
-                const uint32_t oc = tmem + kColY + 128u * (no & 1);
+                const uint32_t oc = tmem + kColO;
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
                     const uint32_t a16 = (kk >> 2) * 512u + (kk & 3) * 2u;    // Y: 8K K-blocks
@@ -571,9 +571,9 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 mbar_arrive(B(B_PF + (g & 1)));
             }
             // row sums to the unit tail; buffer n & 1 was last read by the tail
-            // of unit n - 2 before it released that unit's output
+            // of unit n - 2 before it handed over that unit's Y
             const float lta = quad_sum(la), ltb = quad_sum(lb);
-            if (n >= 2) mbar_wait(B(B_OE + (n & 1)), ((n - 2) >> 1) & 1, status, &abort_flag, 75);
+            if (n >= 2) mbar_wait(B(B_YF + (n & 1)), ((n - 2) >> 1) & 1, status, &abort_flag, 75);
             if (cq == 0) {
                 float *lbuf = reinterpret_cast<float *>(sp + kOffL) + 64 * (n & 1);
                 lbuf[ra] = lta;
@@ -624,7 +624,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             }
             fence_async_smem();
             tc_fence_before();
-            mbar_arrive(B(B_YF));
+            mbar_arrive(B(B_YF + yb));   // Y buffer and row sums read
             const bool ok = mbar_wait(B(B_OF), n & 1, status, &abort_flag, 74);
             tc_fence_after();
             __syncwarp();
@@ -633,7 +633,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
 #pragma unroll 1
             for (int h2 = 0; h2 < 2; ++h2) {
                 uint32_t orr[32];
-                tmem_ld16x256_x8(lbase + ycol + 64u * h2, orr);
+                tmem_ld16x256_x8(lbase + kColO + 64u * h2, orr);
                 tmem_wait_ld();
                 if (ok) {
 #pragma unroll
@@ -649,7 +649,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 }
             }
             tc_fence_before();
-            mbar_arrive(B(B_OE + yb));
+            mbar_arrive(B(B_OE));
             next_unit(sp, it, nu);
             ++n;
         }
