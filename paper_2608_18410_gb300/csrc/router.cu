@@ -30,6 +30,54 @@ __global__ void k_lang_pool(const T *__restrict__ h, const rolesub_episode *__re
     ctx[((size_t)l * E + e) * d + col] = ep.n_lang > 0 ? s / (float)ep.n_lang : 0.f;
 }
 
+// bf16, d % 8 == 0: a thread sums eight adjacent columns (one 16-byte load
+// per row) with four rows in flight; the row order of the sum is the same
+// as above, so the result is too.
+__global__ void k_lang_pool_v8(const __nv_bfloat16 *__restrict__ h, const rolesub_episode *__restrict__ eps, int E,
+                               int64_t rows, int d, float *__restrict__ ctx)
+{
+    const int l = blockIdx.z, e = blockIdx.y;
+    const int c8 = blockIdx.x * blockDim.x + threadIdx.x;
+    if (8 * c8 >= d) return;
+    const rolesub_episode ep = eps[e];
+    const uint4 *base = reinterpret_cast<const uint4 *>(h + ((size_t)l * rows + ep.lang_row_begin) * d) + c8;
+    const size_t stride = (size_t)d / 8;
+    float s[8] = {};
+    const int n = ep.n_lang;
+    int j = 0;
+    for (; j + 4 <= n; j += 4) {
+        uint4 v[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) v[q] = __ldg(base + (size_t)(j + q) * stride);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const __nv_bfloat162 *p = reinterpret_cast<const __nv_bfloat162 *>(&v[q]);
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 f = __bfloat1622float2(p[i]);
+                s[2 * i] += f.x;
+                s[2 * i + 1] += f.y;
+            }
+        }
+    }
+    for (; j < n; ++j) {
+        const uint4 v = __ldg(base + (size_t)j * stride);
+        const __nv_bfloat162 *p = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(p[i]);
+            s[2 * i] += f.x;
+            s[2 * i + 1] += f.y;
+        }
+    }
+    const float fn = (float)n;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s[i] = n > 0 ? s[i] / fn : 0.f;
+    float *out = ctx + ((size_t)l * E + e) * d + 8 * c8;
+    *reinterpret_cast<float4 *>(out) = make_float4(s[0], s[1], s[2], s[3]);
+    *reinterpret_cast<float4 *>(out + 4) = make_float4(s[4], s[5], s[6], s[7]);
+}
+
 // beta[l][e][f] = b1[f] + alpha_lang * W1[f][d+C : 2d+C] . ctx[l][e]
 // A small GEMM per layer (episodes x F x d) in fp32. A cluster of four
 // blocks shares one 64-episode x 32-output tile, each block a quarter of d;
@@ -437,8 +485,12 @@ static cudaError_t launch_router_t(const CompressArgs &a)
     if (M == 0) return cudaSuccess;
     const T *h = (const T *)a.h, *W1 = (const T *)a.W1, *Wre = (const T *)a.W_re,
             *W2 = (const T *)a.W2;
-    k_lang_pool<T><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
-        h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
+    if (sizeof(T) == 2 && d % 8 == 0 && ((uintptr_t)a.h & 15) == 0)
+        k_lang_pool_v8<<<dim3((d / 8 + 127) / 128, E, L), 128, 0, a.stream>>>(
+            (const __nv_bfloat16 *)a.h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
+    else
+        k_lang_pool<T><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
+            h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
     if (sizeof(T) == 2 && d % 128 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
         k_lang_bias_mma<<<dim3((F + 63) / 64 * kMmaSplit, (E + 63) / 64, L), 128, 0, a.stream>>>(
             (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
