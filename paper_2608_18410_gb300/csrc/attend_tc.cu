@@ -29,7 +29,7 @@
 //   Y += P_c Z_c                   tcgen05, M=64, N=128 (rotated space)
 // Unit tail: Y / l -> bf16 smem (a staging tile of its own, so that a Q
 // slot is free as soon as its unit's last S is issued),
-// O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into its own accumulator, output
+// O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into the unit's Y buffer, output
 // stores.
 //
 // Warp roles (512 threads), all hand-offs through mbarriers. Warp w runs on
@@ -43,21 +43,23 @@
 //   warp 7      TMA producer: K (3-slot ring), Q (2 slots), R_h
 //   warps 8-11  unit tail, one per lane quadrant, overlapping the next
 //               unit's chunks (Y is double buffered in TMEM)
-// P is double buffered and Z has four slots: a chunk's softmax waits for the
-// product two chunks back, its gatherer for the one four chunks back, and a
-// gatherer publishes a chunk when it starts its next one.
+// S and P have three buffers and Z four slots: a chunk's S product waits for
+// the softmax three chunks back, its softmax for the P.Z product three chunks
+// back, its gatherer for the one four chunks back, and a gatherer publishes a
+// chunk when it starts its next one.
 //
 // Shared memory (1024-aligned):
 //   0K   Q[2]   16K each (two 64-column K-blocks of 64 rows)
 //   32K  K[3]   16K each (64-row chunks)
 //   80K  Y      16K, Y / l of the unit in its tail (A of the output product)
 //   96K  R_h    32K (two 64-column K-blocks of 128 rows)
-//   128K P[2]   8K each (64 rows x 64 kv)
-//   144K Z[4]   16K each (two 64-column MN-blocks of 64 kv rows)
-//   208K records 4 x 1K
-//   212K row sums 2 x 64 fp32 (softmax -> unit tail)
-//   then the episode table and the barriers
-// TMEM (512 columns): S[2] at 0 and 64, Y[2] at 128 and 256, O at 384.
+//   128K P[3]   8K each (64 rows x 64 kv)
+//   152K Z[4]   16K each (two 64-column MN-blocks of 64 kv rows)
+//   216K records 4 x 1K
+//   220K row sums 2 x 64 fp32 (softmax -> unit tail)
+//   then the unit list and the barriers
+// TMEM (448 of 512 columns): S[3] at 0, 64 and 128, Y[2] at 192 and 320
+// (each later holding its unit's O).
 #include <cuda.h>
 
 #include <algorithm>
@@ -78,7 +80,7 @@ constexpr int kChunk = 64;   // cache tokens per chunk
 constexpr int kQRows = 64;   // query rows per unit
 constexpr int kDh = 128;
 constexpr int kG = 16;       // groups per head (d_s = 8)
-constexpr int kMaxUnits = 448;   // units per CTA and launch (unit list in smem)
+constexpr int kMaxUnits = 256;   // units per CTA and launch (unit list in smem)
 constexpr int kKSlots = 3;
 constexpr float kRescaleLog2 = 8.f;   // raise the reference max beyond 2^8 growth
 
@@ -86,8 +88,9 @@ constexpr uint32_t kOffQ = 0;
 constexpr uint32_t kOffK = 32768;
 constexpr uint32_t kOffY = kOffK + kKSlots * 16384;   // normalised Y of the unit in its tail
 constexpr uint32_t kOffR = 98304;
-constexpr uint32_t kOffP = 131072;
-constexpr uint32_t kOffZ = 147456;                   // 4 x 16K ring
+constexpr int kSBufs = 3;                             // S (TMEM) and P (smem) buffers
+constexpr uint32_t kOffP = 131072;                    // 3 x 8K
+constexpr uint32_t kOffZ = kOffP + kSBufs * 8192;     // 4 x 16K ring
 constexpr int kZSlots = 4;
 constexpr uint32_t kOffRec = kOffZ + kZSlots * 16384; // 4 x 64 x 16 B
 constexpr uint32_t kOffL = kOffRec + 4096;           // 2 x 64 fp32 row sums
@@ -95,7 +98,7 @@ constexpr uint32_t kOffUnits = kOffL + 1024;         // kMaxUnits x 16 B unit re
 constexpr uint32_t kOffBar = kOffUnits + 16 * kMaxUnits;
 constexpr uint32_t kSmemBytes = kOffBar + 512 + 1024;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS = 0, kColY = 128, kColO = 384;   // Y[b] at kColY + 128b
+constexpr uint32_t kColS = 0, kColY = 192;   // S[b] at 64b, Y[b] at kColY + 128b
 
 constexpr uint32_t kIdescS = idesc_bf16(64, 64, false);
 constexpr uint32_t kIdescPV = idesc_bf16(64, 128, true);
@@ -103,8 +106,8 @@ constexpr uint32_t kIdescO = idesc_bf16(64, 128, false);
 
 // barrier slots (8 bytes each); [2] / [4] entries are per buffer
 enum {
-    B_QF = 0, B_QE = 2, B_KF = 4, B_KE = 8, B_RF = 12, B_RE = 13, B_SF = 14, B_PF = 16, B_ZF = 18, B_PV = 22,
-    B_YR = 26, B_YF = 28, B_OF = 30, B_OE = 31, B_LF = 32, B_COUNT = 34
+    B_QF = 0, B_QE = 2, B_KF = 4, B_KE = 8, B_RF = 12, B_RE = 13, B_SF = 14, B_PF = 17, B_ZF = 20, B_PV = 24,
+    B_YR = 28, B_YF = 30, B_OF = 31, B_OE = 32, B_LF = 34, B_COUNT = 36
 };
 
 struct Unit {
@@ -196,7 +199,8 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         abort_flag = 0;
         for (int i = 0; i < B_COUNT; ++i) {
             uint32_t cnt = 1;
-            if (i == B_PF || i == B_PF + 1 || i == B_YF || i == B_YF + 1 || i == B_OE || i == B_LF || i == B_LF + 1)
+            if ((i >= B_PF && i < B_PF + kSBufs) || i == B_YF || i == B_OE || i == B_OE + 1 || i == B_LF ||
+                i == B_LF + 1)
                 cnt = 128;
             if (i >= B_ZF && i < B_ZF + kZSlots) cnt = 64;
             mbar_init(B(i), cnt);
@@ -317,25 +321,27 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         // the start address field, which cannot carry out of its 14 bits
         // below 256 KB). A commit tracks the issuing thread's own products.
         if (lane == 0 && warp == 6) {
-            // S_g = Q K_g^T into S buffer g % 2
+            // S_g = Q K_g^T into S buffer g % 3
             const uint64_t dq = sdesc_sw128(sb + kOffQ, 16, 1024), dk = sdesc_sw128(sb + kOffK, 16, 1024);
             ChunkIt cs = first;
             uint32_t gs = 0, ns = 0;   // chunk counter, unit counter
             while (cs.k < nu) {
                 const uint32_t ks = gs % kKSlots;
-                // S buffer gs % 2 was read by the softmax of chunk gs - 2
-                if (gs >= 2 && !mbar_wait(B(B_PF + (gs & 1)), ((gs - 2) >> 1) & 1, status, &abort_flag, 50)) break;
+                // S buffer gs % 3 was read by the softmax of chunk gs - 3
+                const uint32_t sbuf = gs % kSBufs;
+                if (gs >= kSBufs && !mbar_wait(B(B_PF + sbuf), ((gs / kSBufs) - 1) & 1, status, &abort_flag, 50))
+                    break;
                 if (cs.c == 0 && !mbar_wait(B(B_QF + (ns & 1)), (ns >> 1) & 1, status, &abort_flag, 51)) break;
                 if (!mbar_wait(B(B_KF + ks), (gs / kKSlots) & 1, status, &abort_flag, 52)) break;
                 tc_fence_after();
                 const uint64_t qd = dq + 1024u * (ns & 1), kd = dk + 1024u * ks;
-                const uint32_t sc = tmem + kColS + 64u * (gs & 1);
+                const uint32_t sc = tmem + kColS + 64u * sbuf;
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
                     const uint32_t o16 = (kk >> 2) * 512u + (kk & 3) * 2u;   // (kk/4) * 8K + (kk%4) * 32 bytes
                     mma_bf16(sc, qd + o16, kd + o16, kIdescS, kk > 0);
                 }
-                mma_commit(B(B_SF + (gs & 1)));
+                mma_commit(B(B_SF + sbuf));
                 mma_commit(B(B_KE + ks));
                 if (it_next(sp, cs, nu)) {
                     mma_commit(B(B_QE + (ns & 1)));   // the unit's last S: its Q slot is free
@@ -345,15 +351,15 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             }
         } else if (lane == 0 && warp == 14) {
             // Y += P_g Z_g; a unit's first product starts its Y buffer afresh,
-            // once the tail of the unit two back has read it
+            // once the unit two back has had its output read from it
             const uint64_t dp = sdesc_sw128(sb + kOffP, 16, 1024), dz = sdesc_sw128(sb + kOffZ, 8192, 1024);
             ChunkIt cp = first;
             uint32_t gp = 0, np = 0;
             while (cp.k < nu) {
-                const uint32_t yb = np & 1, b = gp & 1, zs = gp & 3;
-                if (cp.c == 0 && np >= 2 && !mbar_wait(B(B_YF + yb), ((np - 2) >> 1) & 1, status, &abort_flag, 53))
+                const uint32_t yb = np & 1, b = gp % kSBufs, zs = gp & 3;
+                if (cp.c == 0 && np >= 2 && !mbar_wait(B(B_OE + yb), ((np - 2) >> 1) & 1, status, &abort_flag, 53))
                     break;
-                if (!mbar_wait(B(B_PF + b), (gp >> 1) & 1, status, &abort_flag, 54)) break;
+                if (!mbar_wait(B(B_PF + b), (gp / kSBufs) & 1, status, &abort_flag, 54)) break;
                 if (!mbar_wait(B(B_ZF + zs), (gp >> 2) & 1, status, &abort_flag, 55)) break;
                 tc_fence_after();
                 const uint64_t pd = dp + 512u * b, zd = dz + 1024u * zs;
@@ -370,18 +376,17 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 ++gp;
             }
         } else if (lane == 0) {
-            // O = Y R_h^T of each unit, from its normalised Y in shared memory
+            // O = Y R_h^T of each unit, from its normalised Y in shared memory,
+            // written over that unit's Y buffer
             const uint64_t dr = sdesc_sw128(sb + kOffR, 16, 1024), yd = sdesc_sw128(sb + kOffY, 16, 1024);
             ChunkIt co = first;
             uint32_t no = 0;
             int run_o = 0;
             while (co.k < nu) {
-                if (!mbar_wait(B(B_YF + (no & 1)), (no >> 1) & 1, status, &abort_flag, 56)) break;
-                // the O accumulator was read by the tail of the previous unit
-                if (no >= 1 && !mbar_wait(B(B_OE), (no - 1) & 1, status, &abort_flag, 58)) break;
+                if (!mbar_wait(B(B_YF), no & 1, status, &abort_flag, 56)) break;
                 if (!mbar_wait(B(B_RF), run_o & 1, status, &abort_flag, 57)) break;
                 tc_fence_after();
-                const uint32_t oc = tmem + kColO;
+                const uint32_t oc = tmem + kColY + 128u * (no & 1);
 #pragma unroll
                 for (int kk = 0; kk < 8; ++kk) {
                     const uint32_t a16 = (kk >> 2) * 512u + (kk & 3) * 2u;    // Y: 8K K-blocks
@@ -485,11 +490,12 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             float la = 0.f, lb = 0.f;               // this thread's share of the row sums
             for (int c = 0; c < t.nch; ++c, ++g) {
                 const int nk = min(kChunk, t.nc - c * kChunk);
-                mbar_wait(B(B_SF + (g & 1)), (g >> 1) & 1, status, &abort_flag, 70);
+                const uint32_t sbuf = g % kSBufs;
+                mbar_wait(B(B_SF + sbuf), (g / kSBufs) & 1, status, &abort_flag, 70);
                 tc_fence_after();
                 __syncwarp();
                 uint32_t sr[32];
-                tmem_ld16x256_x8(lbase + kColS + 64u * (g & 1), sr);
+                tmem_ld16x256_x8(lbase + kColS + 64u * sbuf, sr);
                 tmem_wait_ld();
                 if (nk < kChunk) {
 #pragma unroll
@@ -552,14 +558,14 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                     pa[j] = pack_bf16(a0, a1);
                     pb[j] = pack_bf16(b0, b1);
                 }
-                // P buffer g & 1 was last read by the product of chunk g - 2
-                if (g >= 2) {
-                    mbar_wait(B(B_PV + ((g - 2) & 3u)), ((g - 2) >> 2) & 1, status, &abort_flag, 72);
+                // P buffer g % 3 was last read by the product of chunk g - 3
+                if (g >= (uint32_t)kSBufs) {
+                    mbar_wait(B(B_PV + ((g - kSBufs) & 3u)), ((g - kSBufs) >> 2) & 1, status, &abort_flag, 72);
                     tc_fence_after();
                 }
                 // 8x8 blocks (rows of ra / rb, 8 columns = one swizzle chunk each):
                 // lane t addresses row t%8 of block t/8
-                const uint32_t prow = sb + kOffP + 8192u * (g & 1) + (uint32_t)(16 * warp + (lane & 7)) * 128u;
+                const uint32_t prow = sb + kOffP + 8192u * sbuf + (uint32_t)(16 * warp + (lane & 7)) * 128u;
                 const uint32_t c0 = ((uint32_t)(lane >> 3) ^ (uint32_t)(lane & 7)) << 4;
                 const uint32_t c1 = ((uint32_t)((lane >> 3) + 4) ^ (uint32_t)(lane & 7)) << 4;
                 stmatrix_x4(prow + c0, pa[0], pa[1], pa[2], pa[3]);
@@ -568,12 +574,12 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 stmatrix_x4(prow + 1024u + c1, pb[4], pb[5], pb[6], pb[7]);
                 fence_async_smem();
                 tc_fence_before();
-                mbar_arrive(B(B_PF + (g & 1)));
+                mbar_arrive(B(B_PF + sbuf));
             }
             // row sums to the unit tail; buffer n & 1 was last read by the tail
-            // of unit n - 2 before it handed over that unit's Y
+            // of unit n - 2 before it released that unit's output
             const float lta = quad_sum(la), ltb = quad_sum(lb);
-            if (n >= 2) mbar_wait(B(B_YF + (n & 1)), ((n - 2) >> 1) & 1, status, &abort_flag, 75);
+            if (n >= 2) mbar_wait(B(B_OE + (n & 1)), ((n - 2) >> 1) & 1, status, &abort_flag, 75);
             if (cq == 0) {
                 float *lbuf = reinterpret_cast<float *>(sp + kOffL) + 64 * (n & 1);
                 lbuf[ra] = lta;
@@ -624,7 +630,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             }
             fence_async_smem();
             tc_fence_before();
-            mbar_arrive(B(B_YF + yb));   // Y buffer and row sums read
+            mbar_arrive(B(B_YF));
             const bool ok = mbar_wait(B(B_OF), n & 1, status, &abort_flag, 74);
             tc_fence_after();
             __syncwarp();
@@ -633,7 +639,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
 #pragma unroll 1
             for (int h2 = 0; h2 < 2; ++h2) {
                 uint32_t orr[32];
-                tmem_ld16x256_x8(lbase + kColO + 64u * h2, orr);
+                tmem_ld16x256_x8(lbase + ycol + 64u * h2, orr);
                 tmem_wait_ld();
                 if (ok) {
 #pragma unroll
@@ -649,7 +655,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 }
             }
             tc_fence_before();
-            mbar_arrive(B(B_OE));
+            mbar_arrive(B(B_OE + yb));
             next_unit(sp, it, nu);
             ++n;
         }
