@@ -103,7 +103,9 @@ static __device__ __noinline__ void wait_timed_out(int32_t *status, volatile int
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status,
                                           volatile int *abort, int where)
 {
-    if (mbar_try_wait_sleep(bar, parity, kSleepHintNs)) return true;
+    // a phase that has already completed costs one non-blocking test (a
+    // try_wait with a suspend hint costs several times more even then)
+    if (mbar_test(bar, parity)) return true;
     const uint64_t t0 = global_ns();
 #pragma unroll 1
     for (;;) {
