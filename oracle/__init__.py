@@ -13,6 +13,9 @@ Parity status of each function (what pins it, in tests/test_oracle_pins.py):
   lang_pool       -- closed form (mean), empty-set case
   role            -- scipy.special.softmax, uniform case
   router_score    -- one-block-at-a-time special cases (h / role / language)
+  router_score_linear -- the additive form: selector-matrix closed forms for
+                     each term, one term at a time and together; parameter
+                     count against the paper's 4.20M routing heads
   topk            -- brute-force subset enumeration, hand-built near-ties
   rotate          -- permutation matrices, norm preservation
   compress/attend -- all-kept == dense attention (1e-10), none-kept == 0,
@@ -65,6 +68,11 @@ def lib():
             L.oracle_role.restype = None
             L.oracle_router_score.argtypes = [ctypes.c_int] * 4 + [_dp] * 7 + [ctypes.c_double] * 2 + [_dp]
             L.oracle_router_score.restype = None
+            L.oracle_router_score_linear.argtypes = [ctypes.c_int] * 3 + [_dp] * 8 + [ctypes.c_double] * 2 + [_dp]
+            L.oracle_router_score_linear.restype = None
+            L.oracle_route_episode_linear.argtypes = (
+                [ctypes.c_int] * 3 + [_ip, _ip, _llp] + [_dp] * 8 + [ctypes.c_double] * 2 + [_ubp, _dp, _dp])
+            L.oracle_route_episode_linear.restype = ctypes.c_int
             L.oracle_topk.argtypes = [ctypes.c_int, ctypes.c_int, _dp, _ubp, _dp]
             L.oracle_topk.restype = None
             L.oracle_rotate.argtypes = [ctypes.c_int, _dp, _dp, _dp]
@@ -162,6 +170,25 @@ def router_score(W1, b1, W2, b2, h, a, c, alpha_role, alpha_lang):
     return g
 
 
+def router_score_linear(W_v, b_v, W_role, W_l, b_l, h, a, c, alpha_role, alpha_lang):
+    """Additive router (Eq. routingscore as printed) for one token."""
+    W_v, wv = _d(W_v)
+    b_v, bv = _d(b_v)
+    W_role, wr = _d(W_role)
+    W_l, wl = _d(W_l)
+    b_l, bl = _d(b_l)
+    h, hp = _d(h)
+    a, ap = _d(a)
+    c, cp = _d(c)
+    G, d = W_v.shape
+    C = a.shape[0]
+    assert W_l.shape == (G, d) and W_role.shape == (G, C) and h.shape[0] == d
+    g = np.zeros(G)
+    lib().oracle_router_score_linear(d, C, G, wv, bv, wr, wl, bl, hp, ap, cp, float(alpha_role),
+                                     float(alpha_lang), g.ctypes.data_as(_dp))
+    return g
+
+
 def topk(gamma, k):
     gamma, gp = _d(gamma)
     G = gamma.shape[0]
@@ -249,6 +276,48 @@ def compress_layer(spec: Spec, h, v, R, W_re, b_re, W1, b1, W2, b2, alpha_role, 
         if want_z:
             z[r0:r1] = z_e[:r1 - r0]
     return {"packed": packed, "idx": idx[:lay["idx_bytes"]], "gamma": gamma, "margin": margin, "z": z}
+
+
+def compress_layer_linear(spec: Spec, h, v, R, W_re, b_re, W_v, b_v, W_role, W_l, b_l, alpha_role, alpha_lang,
+                          episodes=None, want_z=True):
+    """Compress one layer with the additive router: route every (listed)
+    episode, then rotate and pack with those indices (compress_layer with
+    idx_force). Same return dict as compress_layer."""
+    s = spec
+    lay = s.lay
+    idx = np.zeros(max(lay["idx_bytes"], 1), np.uint8)
+    gamma = np.full((lay["rows"], s.G), np.nan)
+    margin = np.full(lay["rows"], np.nan)
+    Wre, Wrep = _d(W_re)
+    bre, brep = _d(b_re)
+    Wv, Wvp = _d(W_v)
+    bv, bvp = _d(b_v)
+    Wr, Wrp = _d(W_role)
+    Wl, Wlp = _d(W_l)
+    bl, blp = _d(b_l)
+    eps = list(range(s.E)) if episodes is None else list(episodes)
+    for e in eps:
+        r0, r1 = int(s.ep_row[e]), int(s.ep_row[e + 1])
+        he, hp = _d(h[r0:r1] if r1 > r0 else np.zeros((1, s.d)))
+        nt, ntp = _i(s.n_tok[e])
+        kk, kp = _i(s.k[e])
+        io, iop = _ll(lay["idx_off"][4 * e:4 * e + 4])
+        g_e = np.full((max(r1 - r0, 1), s.G), np.nan)
+        m_e = np.full(max(r1 - r0, 1), np.nan)
+        rc = lib().oracle_route_episode_linear(
+            s.d, s.G, s.C, ntp, kp, iop, hp, Wrep, brep, Wvp, bvp, Wrp, Wlp, blp,
+            float(alpha_role), float(alpha_lang), _u8(idx), g_e.ctypes.data_as(_dp), m_e.ctypes.data_as(_dp))
+        if rc != 0:
+            raise ValueError("oracle_route_episode_linear: bad arguments")
+        gamma[r0:r1] = g_e[:r1 - r0]
+        margin[r0:r1] = m_e[:r1 - r0]
+    # rotation and packing with the routed indices (router weights unused there)
+    zF = np.zeros((1, 2 * s.d + s.C))
+    out = compress_layer(spec, h, v, R, W_re, b_re, zF, np.zeros(1), np.zeros((s.G, 1)), np.zeros(s.G),
+                         alpha_role, alpha_lang, episodes=eps, idx_force=idx, want_z=want_z)
+    out["gamma"] = gamma
+    out["margin"] = margin
+    return out
 
 
 def attend_layer(spec: Spec, q, K, packed, idx, R, scale=0.0, episodes=None, heads=None, out=None):

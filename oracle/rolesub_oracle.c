@@ -17,7 +17,9 @@
  *             uses the concatenation form gamma = W2 ReLU(W1 [h; a_r a; a_l c]
  *             + b1) + b2 with c the mean of the episode's retained language
  *             hidden states; the K_i largest scores are kept (ties: lower
- *             group index first).
+ *             group index first). oracle_router_score_linear is the
+ *             additive form as printed (linear f_v and f_lang heads, W_role
+ *             a, each term weighted as in the equation).
  *   Attention (Sec. 3, keys and queries unchanged; values routed):
  *             s_j = q . k_j * scale, p = softmax_j(s) over every cache token
  *             of the episode (non-causal), o = sum_j p_j v~_j, evaluated as
@@ -124,6 +126,30 @@ void oracle_router_score(int d, int C, int F, int G,
     }
     free(x);
     free(u);
+}
+
+/* Eq. (routingscore) as printed, the additive form, with linear scoring
+ * heads (the paper leaves f_v and f_lang as "learned scoring functions"):
+ *   gamma_token = W_v h + b_v            W_v is [G][d]
+ *   gamma_role  = W_role a               W_role is [G][C], no bias
+ *   gamma_lang  = W_l c + b_l            W_l is [G][d], c the pooled context
+ *   gamma = gamma_token + alpha_role gamma_role + alpha_lang gamma_lang      */
+void oracle_router_score_linear(int d, int C, int G,
+                                const double *W_v, const double *b_v,
+                                const double *W_role,
+                                const double *W_l, const double *b_l,
+                                const double *h, const double *a, const double *c,
+                                double alpha_role, double alpha_lang, double *gamma)
+{
+    for (int g = 0; g < G; ++g) {
+        double tok = b_v[g];
+        for (int t = 0; t < d; ++t) tok += W_v[(size_t)g * d + t] * h[t];
+        double role = 0.0;
+        for (int r = 0; r < C; ++r) role += W_role[(size_t)g * C + r] * a[r];
+        double lang = b_l[g];
+        for (int t = 0; t < d; ++t) lang += W_l[(size_t)g * d + t] * c[t];
+        gamma[g] = tok + alpha_role * role + alpha_lang * lang;
+    }
 }
 
 /* Top-K_i of Sec. 3.4. Groups are ranked by (gamma descending, index
@@ -256,6 +282,63 @@ int oracle_compress_episode(int H, int dh, int G, int C, int F,
     free(gam);
     free(z);
     return rc;
+}
+
+/*
+ * Routing of one episode of one layer with the additive router above:
+ * c = pool of the language rows, then for every token of a segment with
+ * 0 < k < G the top-k of gamma (Sec. 3.4); k = G keeps every group in order.
+ * Writes the layer's index array at the segment offsets, and optionally
+ * gamma_ep [n_cache][G] (NaN where the router does not run) and margin_ep.
+ * The packing that follows is oracle_compress_episode with these indices.
+ * Returns 0, or -1 on bad arguments.
+ */
+int oracle_route_episode_linear(int d, int G, int C, const int *n_tok, const int *k,
+                                const long long *idx_off, const double *h_ep,
+                                const double *W_re, const double *b_re,
+                                const double *W_v, const double *b_v, const double *W_role,
+                                const double *W_l, const double *b_l,
+                                double alpha_role, double alpha_lang,
+                                unsigned char *idx_layer, double *gamma_ep, double *margin_ep)
+{
+    if (d <= 0 || G <= 0 || G > 64 || C < 0) return -1;
+    int row0[OR_KINDS];
+    int nc = 0;
+    for (int m = 0; m < OR_KINDS; ++m) {
+        if (n_tok[m] < 0 || k[m] < 0 || k[m] > G) return -1;
+        row0[m] = nc;
+        nc += n_tok[m];
+    }
+    double *c = (double *)malloc(sizeof(double) * (size_t)d);
+    oracle_lang_pool(d, n_tok[1], h_ep + (size_t)row0[1] * d, c);
+    double *a = (double *)malloc(sizeof(double) * (size_t)(C > 0 ? C : 1));
+    double *gam = (double *)malloc(sizeof(double) * (size_t)G);
+    for (int m = 0; m < OR_KINDS; ++m) {
+        int n = n_tok[m], kk = k[m];
+        for (int i = 0; i < n; ++i) {
+            int r = row0[m] + i;
+            const double *h = h_ep + (size_t)r * d;
+            unsigned char *ix = idx_layer + idx_off[m] + (long long)i * kk;
+            double mg = INFINITY;
+            if (gamma_ep)
+                for (int g = 0; g < G; ++g) gamma_ep[(size_t)r * G + g] = NAN;
+            if (kk == G) {
+                for (int j = 0; j < G; ++j) ix[j] = (unsigned char)j;
+            } else if (kk > 0) {
+                oracle_role(d, C, W_re, b_re, h, a);
+                oracle_router_score_linear(d, C, G, W_v, b_v, W_role, W_l, b_l, h, a, c,
+                                           alpha_role, alpha_lang, gam);
+                oracle_topk(G, kk, gam, ix, &mg);
+                if (gamma_ep)
+                    for (int g = 0; g < G; ++g) gamma_ep[(size_t)r * G + g] = gam[g];
+            }
+            if (margin_ep) margin_ep[r] = mg;
+        }
+    }
+    free(c);
+    free(a);
+    free(gam);
+    return 0;
 }
 
 /*

@@ -479,3 +479,108 @@ def test_bad_forced_indices_rejected(oracle):
         run(oracle, p, idx_force=np.array([0, 4, 1, 2], np.uint8))   # 4 >= G
     with pytest.raises(ValueError):
         run(oracle, p, idx_force=np.array([1, 1, 1, 2], np.uint8))   # not ascending
+
+
+# ---------------------------------------------------------------------------
+# Additive router (Eq. routingscore as printed, linear scoring heads)
+# ---------------------------------------------------------------------------
+
+def test_additive_router_parameter_count_matches_paper():
+    # two linear S x d heads with biases (f_v, f_lang) and the S x C role
+    # projection, per layer, 32 layers, S = 16, d = 4096, C = 6: the paper
+    # reports about 4.20M routing-head parameters (Sec. 4, implementation)
+    S, d, C, L = 16, 4096, 6, 32
+    per_layer = 2 * (S * d + S) + S * C
+    assert round(per_layer * L / 1e6, 2) == 4.20
+
+
+def _selectors(rng, G, d):
+    perm = rng.permutation(d)[:G]
+    W = np.zeros((G, d))
+    W[np.arange(G), perm] = 1.0
+    return W, perm
+
+
+def test_additive_router_token_term_alone(oracle):
+    rng = np.random.default_rng(30)
+    d, G, C = 10, 4, 3
+    W_v, perm = _selectors(rng, G, d)
+    b_v = rng.standard_normal(G)
+    h = rng.standard_normal(d)
+    g = oracle.router_score_linear(W_v, b_v, rng.standard_normal((G, C)), rng.standard_normal((G, d)),
+                                   rng.standard_normal(G), h, rng.random(C), rng.standard_normal(d), 0.0, 0.0)
+    assert np.array_equal(g, h[perm] + b_v)
+
+
+def test_additive_router_role_term_alone(oracle):
+    rng = np.random.default_rng(31)
+    d, G, C = 10, 6, 3
+    # row s of W_role picks role s mod C with weight w_s
+    w = rng.standard_normal(G)
+    W_role = np.zeros((G, C))
+    W_role[np.arange(G), np.arange(G) % C] = w
+    a = rng.random(C)
+    g = oracle.router_score_linear(np.zeros((G, d)), np.zeros(G), W_role, np.zeros((G, d)), np.zeros(G),
+                                   rng.standard_normal(d), a, rng.standard_normal(d), 0.25, 0.7)
+    assert np.max(np.abs(g - 0.25 * w * a[np.arange(G) % C])) < 1e-16
+
+
+def test_additive_router_language_term_alone(oracle):
+    rng = np.random.default_rng(32)
+    d, G, C = 10, 4, 3
+    W_l, perm = _selectors(rng, G, d)
+    b_l = rng.standard_normal(G)
+    h_lang = rng.standard_normal((5, d))
+    c = oracle.lang_pool(h_lang)
+    g = oracle.router_score_linear(np.zeros((G, d)), np.zeros(G), rng.standard_normal((G, C)), W_l, b_l,
+                                   rng.standard_normal(d), rng.random(C), c, 0.0, 0.125)
+    # the language weight scales the head's bias too: alpha_lang * (W_l c + b_l)
+    assert np.max(np.abs(g - 0.125 * (h_lang.mean(0)[perm] + b_l))) < 1e-15
+
+
+def test_additive_router_terms_add(oracle):
+    rng = np.random.default_rng(33)
+    d, G, C = 12, 4, 3
+    W_v, pv = _selectors(rng, G, d)
+    W_l, pl = _selectors(rng, G, d)
+    w = rng.standard_normal(G)
+    W_role = np.zeros((G, C))
+    W_role[np.arange(G), np.arange(G) % C] = w
+    b_v, b_l = rng.standard_normal(G), rng.standard_normal(G)
+    h, c, a = rng.standard_normal(d), rng.standard_normal(d), rng.random(C)
+    g = oracle.router_score_linear(W_v, b_v, W_role, W_l, b_l, h, a, c, -0.3, 0.6)
+    want = (h[pv] + b_v) - 0.3 * w * a[np.arange(G) % C] + 0.6 * (c[pl] + b_l)
+    assert np.max(np.abs(g - want)) < 1e-15
+
+
+def test_additive_router_compress_keeps_best_subset_and_packs_rotated_groups(oracle):
+    rng = np.random.default_rng(34)
+    H, dh, G, C = 2, 8, 4, 3
+    d = H * dh
+    n_tok, k = ((6, 3, 0, 0),), ((2, 1, G, G),)
+    p = rnd_problem(rng, H=H, dh=dh, G=G, C=C, F=4, n_tok=n_tok, k=k, n_q=(1,))
+    spec = oracle.Spec(H, dh, G, C, 4, p["n_tok"], p["k"], p["n_q"])
+    W_v, pv = _selectors(rng, G, d)
+    W_role = rng.standard_normal((G, C))
+    W_l, pl = _selectors(rng, G, d)
+    b_v, b_l = rng.standard_normal(G), rng.standard_normal(G)
+    out = oracle.compress_layer_linear(spec, p["h"], p["v"], p["R"], p["W_re"], p["b_re"], W_v, b_v, W_role,
+                                       W_l, b_l, 0.2, 0.4)
+    cl = p["h"][6:9].mean(0)
+    lay = spec.lay
+    ds = dh // G
+    for r in range(9):
+        kk = 2 if r < 6 else 1
+        a = scipy.special.softmax(p["W_re"] @ p["h"][r] + p["b_re"])
+        gam = (p["h"][r][pv] + b_v) + 0.2 * (W_role @ a) + 0.4 * (cl[pl] + b_l)
+        assert np.max(np.abs(out["gamma"][r] - gam)) < 1e-12
+        best = max(itertools.combinations(range(G), kk), key=lambda s: sum(gam[list(s)]))
+        m, i = (0, r) if r < 6 else (1, r - 6)
+        sel = out["idx"][lay["idx_off"][m] + i * kk:lay["idx_off"][m] + (i + 1) * kk]
+        assert tuple(sel) == tuple(sorted(best))
+        n = 6 if r < 6 else 3
+        for hh in range(H):
+            z = p["R"][hh].T @ p["v"][r, hh * dh:(hh + 1) * dh]
+            base = lay["packed_off"][m] + ((hh * n + i) * kk) * ds
+            want = np.concatenate([z[g * ds:(g + 1) * ds] for g in sel])
+            assert np.max(np.abs(out["packed"][base:base + kk * ds] - want)) < 1e-12
