@@ -189,6 +189,32 @@ rolesub_status rolesub_compress(const rolesub_shape *shape, const void *plan_hos
                                 size_t ws_bytes, void *stream);
 
 /*
+ * rolesub_compress with the routing score in the additive form of Sec. 3.4
+ * (Eq. routingscore), the token and language heads being linear maps:
+ *   gamma_i = (W_v h_i + b_v) + alpha_role W_role a_i
+ *             + alpha_lang (W_l c_e + b_l)
+ *   a_i = softmax(W_re h_i + b_re)            Eq. (latentrole)
+ *   c_e = mean of the episode's retained language hidden states (Sec. 3.4)
+ * then the K_i largest gamma are kept (ties: lower group index) and the
+ * rotation and packing run exactly as in rolesub_compress.
+ * Inputs (device, dtype = shape.dtype unless noted, row-major contiguous):
+ *   h, v, R, W_re, b_re     as rolesub_compress
+ *   W_v    [L][S][d], b_v [L][S] float32     token head
+ *   W_role [L][S][C]                          role head
+ *   W_l    [L][S][d], b_l [L][S] float32     language head
+ * shape.router_hidden is not used by this call (any value >= 1).
+ * Outputs, workspace (rolesub_workspace_size of the same shape), stream and
+ * errors: as rolesub_compress; ROLESUB_EUNSUPPORTED when S > 32 or C > 4096.
+ */
+rolesub_status rolesub_compress_additive(const rolesub_shape *shape, const void *plan_host,
+                                         const void *plan_dev, const void *h, const void *v,
+                                         const void *R, const void *W_re, const float *b_re,
+                                         const void *W_v, const float *b_v, const void *W_role,
+                                         const void *W_l, const float *b_l, float alpha_role,
+                                         float alpha_lang, void *packed_v, uint8_t *idx,
+                                         void *workspace, size_t ws_bytes, void *stream);
+
+/*
  * Attention of every episode's query tokens over its own routed cache
  * (all cache tokens of the episode, non-causal), per layer and head:
  *   s_j = (q . k_j) * scale, p = softmax_j(s), y = sum_j p_j M_j z_j,

@@ -97,7 +97,11 @@ WsSizes ws_sizes(const rolesub_shape *s, const rolesub_plan *p)
     const size_t d = (size_t)s->num_heads * s->head_dim;
     w.status = rs::kStatusBytes;
     w.ctx = align_up(sizeof(float) * L * E * d, kAlign);
-    w.bias = align_up(sizeof(float) * L * E * s->router_hidden, kAlign);
+    // per-episode router terms: F wide for the concatenation router, S for
+    // the additive one
+    w.bias = align_up(sizeof(float) * L * E * (size_t)(s->router_hidden > s->num_groups ? s->router_hidden
+                                                                                      : s->num_groups),
+                      kAlign);
     // router logits are only staged in memory when the fused tensor-core
     // router does not apply
     w.logits = rs::router_tc_supported(s)
@@ -314,6 +318,49 @@ rolesub_status rolesub_compress(const rolesub_shape *shape, const void *plan_hos
     a.idx = idx;
     a.stream = (cudaStream_t)stream;
     cudaError_t e = rs::launch_router(a);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    return from_cuda(rs::launch_rotate_pack(a));
+}
+
+rolesub_status rolesub_compress_additive(const rolesub_shape *shape, const void *plan_host,
+                                         const void *plan_dev, const void *h, const void *v,
+                                         const void *R, const void *W_re, const float *b_re,
+                                         const void *W_v, const float *b_v, const void *W_role,
+                                         const void *W_l, const float *b_l, float alpha_role,
+                                         float alpha_lang, void *packed_v, uint8_t *idx,
+                                         void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!shape_ok(shape)) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, plan_dev, &pv);
+    if (st != ROLESUB_OK) return st;
+    if (!plan_dev) return ROLESUB_EINVAL;
+    const void *ptrs[] = {h, v, R, W_re, b_re, W_v, b_v, W_role, W_l, b_l, workspace};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    const rolesub_plan &P = *pv.hdr;
+    if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
+    if (P.idx_bytes_per_layer > 0 && (!idx || !aligned16(idx))) return ROLESUB_EINVAL;
+    if (!isfinite(alpha_role) || !isfinite(alpha_lang)) return ROLESUB_EINVAL;
+    const WsSizes w = ws_sizes(shape, pv.hdr);
+    if (ws_bytes < w.total) return ROLESUB_EINVAL;
+    if (!rs::router_additive_supported(shape) || !rs::rotate_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    rs::CompressArgs a{};
+    a.shape = shape;
+    a.plan = pv;
+    a.ws = carve(w, workspace);
+    a.h = h;
+    a.v = v;
+    a.R = R;
+    a.W_re = W_re;
+    a.b_re = b_re;
+    a.alpha_role = alpha_role;
+    a.alpha_lang = alpha_lang;
+    a.packed = packed_v;
+    a.idx = idx;
+    a.stream = (cudaStream_t)stream;
+    const rs::AdditiveWeights wt{W_v, W_role, W_l, b_v, b_l};
+    cudaError_t e = rs::launch_router_additive(a, wt);
     if (e != cudaSuccess) return ROLESUB_ECUDA;
     return from_cuda(rs::launch_rotate_pack(a));
 }

@@ -45,6 +45,14 @@ struct CompressArgs {
     cudaStream_t stream;
 };
 
+// Weights of the additive routing score (Sec. 3.4, Eq. routingscore):
+// W_v, W_l [L][S][d] and W_role [L][S][C] in the shape's dtype, b_v, b_l
+// [L][S] float32.
+struct AdditiveWeights {
+    const void *W_v, *W_role, *W_l;
+    const float *b_v, *b_l;
+};
+
 struct AttendArgs {
     const rolesub_shape *shape;
     PlanView plan;
@@ -59,6 +67,12 @@ struct AttendArgs {
 
 // Router: language pool + per-episode bias, router GEMM, epilogue/top-k.
 cudaError_t launch_router(const CompressArgs &a);
+// Language pool c_e of every (layer, episode) into ws.lang_ctx.
+cudaError_t launch_lang_pool(const CompressArgs &a);
+// Additive router: language term per episode, then scores and top-k per
+// routed row (tcgen05 for bf16, S = 16, S + C <= 256, d % 64 == 0).
+bool router_additive_supported(const rolesub_shape *s);
+cudaError_t launch_router_additive(const CompressArgs &a, const AdditiveWeights &w);
 // Rotation z = R_h^T v and packing of the kept groups.
 cudaError_t launch_rotate_pack(const CompressArgs &a);
 // Fused router GEMM + epilogue + top-k on tcgen05/TMA (bf16, F = 256,

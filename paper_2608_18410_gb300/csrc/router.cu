@@ -474,6 +474,24 @@ bool router_supported(const rolesub_shape *s)
     return s->role_dim + s->router_hidden <= 1536 && s->num_groups <= 32;
 }
 
+cudaError_t launch_lang_pool(const CompressArgs &a)
+{
+    const rolesub_shape &S = *a.shape;
+    const rolesub_plan &P = *a.plan.hdr;
+    const int L = S.num_layers, E = P.num_episodes, d = S.num_heads * S.head_dim;
+    if (S.dtype == ROLESUB_BF16 && d % 8 == 0 && ((uintptr_t)a.h & 15) == 0)
+        k_lang_pool_v8<<<dim3((d / 8 + 127) / 128, E, L), 128, 0, a.stream>>>(
+            (const __nv_bfloat16 *)a.h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
+    else if (S.dtype == ROLESUB_BF16)
+        k_lang_pool<__nv_bfloat16><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
+            (const __nv_bfloat16 *)a.h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
+    else
+        k_lang_pool<float><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
+            (const float *)a.h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
+    count_launches(1);
+    return cudaGetLastError();
+}
+
 template <class T>
 static cudaError_t launch_router_t(const CompressArgs &a)
 {
@@ -485,12 +503,8 @@ static cudaError_t launch_router_t(const CompressArgs &a)
     if (M == 0) return cudaSuccess;
     const T *h = (const T *)a.h, *W1 = (const T *)a.W1, *Wre = (const T *)a.W_re,
             *W2 = (const T *)a.W2;
-    if (sizeof(T) == 2 && d % 8 == 0 && ((uintptr_t)a.h & 15) == 0)
-        k_lang_pool_v8<<<dim3((d / 8 + 127) / 128, E, L), 128, 0, a.stream>>>(
-            (const __nv_bfloat16 *)a.h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
-    else
-        k_lang_pool<T><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
-            h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
+    cudaError_t err = launch_lang_pool(a);
+    if (err != cudaSuccess) return err;
     if (sizeof(T) == 2 && d % 128 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
         k_lang_bias_mma<<<dim3((F + 63) / 64 * kMmaSplit, (E + 63) / 64, L), 128, 0, a.stream>>>(
             (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
@@ -498,7 +512,7 @@ static cudaError_t launch_router_t(const CompressArgs &a)
         k_lang_bias<T><<<dim3((F + 31) / 32 * kBiasSplit, (E + 63) / 64, L), 256, 0, a.stream>>>(
             W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
     if (router_tc_supported(a.shape)) {
-        count_launches(2);
+        count_launches(1);
         cudaError_t e = cudaGetLastError();
         return e != cudaSuccess ? e : launch_router_tc(a);
     }
@@ -510,7 +524,7 @@ static cudaError_t launch_router_t(const CompressArgs &a)
     k_router_epilogue<T><<<dim3((unsigned)((M + 7) / 8), L), 256, smem, a.stream>>>(
         a.ws.logits, pd, M, d, C, F, G, E, W1, a.ws.lang_bias, W2, a.b2, a.alpha_role, a.idx,
         P.idx_bytes_per_layer);
-    count_launches(4);
+    count_launches(3);
     return cudaGetLastError();
 }
 

@@ -30,7 +30,7 @@ STATUS = {0: "ROLESUB_OK", 1: "ROLESUB_EINVAL", 2: "ROLESUB_EUNSUPPORTED", 3: "R
 EXPORTS = ("rolesub_plan_size", "rolesub_layout_plan", "rolesub_workspace_size",
            "rolesub_compress", "rolesub_attend", "rolesub_get_device_status",
            "rolesub_reset_device_status", "rolesub_status_string", "rolesub_version",
-           "rolesub_launch_count", "rolesub_compress_static")
+           "rolesub_launch_count", "rolesub_compress_static", "rolesub_compress_additive")
 
 STATIC_SCRATCH_BYTES = 8 << 20
 
@@ -108,6 +108,8 @@ def lib():
         L.rolesub_version.restype = ctypes.c_int32
         L.rolesub_compress_static.argtypes = ([sp, _vp, _vp] + [_vp] * 9 + [ctypes.c_float, ctypes.c_float]
                                               + [_vp, _vp, _vp])
+        L.rolesub_compress_additive.argtypes = ([sp, _vp, _vp] + [_vp] * 10 + [ctypes.c_float, ctypes.c_float]
+                                                + [_vp, _vp, _vp, ctypes.c_size_t, _vp])
         L.rolesub_launch_count.argtypes = []
         L.rolesub_launch_count.restype = ctypes.c_uint64
         for name in EXPORTS:
@@ -204,6 +206,15 @@ def rolesub_compress(shape, plan: Plan, plan_dev, h, v, R, W_re, b_re, W1, b1, W
         _ptr(packed_v), _ptr(idx), _ptr(workspace), int(ws_bytes), _stream(stream)))
 
 
+def rolesub_compress_additive(shape, plan: Plan, plan_dev, h, v, R, W_re, b_re, W_v, b_v, W_role, W_l, b_l,
+                              alpha_role, alpha_lang, packed_v, idx, workspace, ws_bytes=None, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size() if ws_bytes is None else ws_bytes
+    _check("rolesub_compress_additive", lib().rolesub_compress_additive(
+        ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(h), _ptr(v), _ptr(R), _ptr(W_re),
+        _ptr(b_re), _ptr(W_v), _ptr(b_v), _ptr(W_role), _ptr(W_l), _ptr(b_l), float(alpha_role),
+        float(alpha_lang), _ptr(packed_v), _ptr(idx), _ptr(workspace), int(ws_bytes), _stream(stream)))
+
+
 def rolesub_attend(shape, plan: Plan, plan_dev, q, q_strides, K, k_strides, packed_v, idx, R,
                    softmax_scale, o, workspace, ws_bytes=None, stream=None):
     ws_bytes = workspace.numel() * workspace.element_size() if ws_bytes is None else ws_bytes
@@ -284,6 +295,15 @@ class RoleSub:
             packed, idx = self.new_outputs()
         rolesub_compress(self.shape, self.plan, self.plan_dev, h, v, R, W_re, b_re, W1, b1, W2, b2,
                          alpha_role, alpha_lang, packed, idx, self.workspace, self.ws_bytes, stream)
+        return packed, idx
+
+    def compress_additive(self, h, v, R, W_re, b_re, W_v, b_v, W_role, W_l, b_l, alpha_role=0.1,
+                          alpha_lang=0.1, packed=None, idx=None, stream=None):
+        if packed is None or idx is None:
+            packed, idx = self.new_outputs()
+        rolesub_compress_additive(self.shape, self.plan, self.plan_dev, h, v, R, W_re, b_re, W_v, b_v, W_role,
+                                  W_l, b_l, alpha_role, alpha_lang, packed, idx, self.workspace, self.ws_bytes,
+                                  stream)
         return packed, idx
 
     def attend(self, q, K, packed, idx, R, softmax_scale=0.0, o=None, q_strides=None, k_strides=None,

@@ -12,6 +12,8 @@ Recipe (one numpy PCG64 stream per tensor block):
   activations h, v, q, K   ~ N(0, 1)      drawn in float32
   weights W_re, W1, W2     ~ N(0, 0.02)   drawn in float32, scaled in float32
   biases  b_re, b1, b2     ~ N(0, 0.02)   float32 (biases are always fp32)
+  additive router (gen_additive_weights):
+    W_v, W_l ~ N(0, 0.02), W_role ~ N(0, 1), b_v, b_l ~ N(0, 0.02) (fp32)
   R_h: Haar-random orthogonal d_h x d_h, from the QR factorisation of an
        fp64 N(0, 1) matrix with column signs fixed by sign(diag(R_qr)).
 bf16 tensors are rounded float32 -> bf16 with round-to-nearest-even and are
@@ -31,7 +33,7 @@ KINDS = ("vis", "lang", "prop", "act")
 
 TID = {"h": 1, "v": 2, "q": 3, "K": 4, "R": 5, "W_re": 6, "b_re": 7,
        "W1": 8, "b1": 9, "W2": 10, "b2": 11, "episodes": 12, "near_tie": 13,
-       "packed": 14, "idx": 15}
+       "packed": 14, "idx": 15, "W_v": 16, "b_v": 17, "W_role": 18, "W_l": 19, "b_l": 20}
 
 
 @dataclasses.dataclass(frozen=True)
@@ -291,6 +293,43 @@ def gen_inputs(wl: Workload, threads: int = 8):
             jobs.append(ex.submit(_fill_layer_acts, wl, out, layer))
         for j in jobs:
             j.result()
+    return out
+
+
+def gen_additive_weights(wl: Workload):
+    """Token, role and language heads of the additive routing score, every layer.
+
+    W_v, W_l [L][G][d] and W_role [L][G][C] in the workload's storage dtype;
+    b_v, b_l [L][G] float32. W_role is drawn at unit scale: it maps a
+    probability vector, so its term is comparable to the others at
+    alpha_role = 0.1. With wl.near_tie, groups form clusters of 4 with
+    identical rows of W_v, W_role, W_l and b_l, and b_v as in the
+    concatenation router's near-tie recipe (cluster 0 tied exactly, the others
+    offset by uniform [0, 1e-3)).
+    """
+    s, d, G, C, L = wl.seed, wl.d, wl.G, wl.C, wl.L
+    sd = storage_dtype(wl.dtype)
+    out = {"W_v": np.empty((L, G, d), sd), "b_v": np.empty((L, G), np.float32),
+           "W_role": np.empty((L, G, C), sd), "W_l": np.empty((L, G, d), sd),
+           "b_l": np.empty((L, G), np.float32)}
+    for layer in range(L):
+        Wv = _normal(s, layer, 0, TID["W_v"], (G, d), 0.02)
+        bv = _normal(s, layer, 0, TID["b_v"], (G,), 0.02)
+        Wr = _normal(s, layer, 0, TID["W_role"], (G, C))
+        Wl = _normal(s, layer, 0, TID["W_l"], (G, d), 0.02)
+        bl = _normal(s, layer, 0, TID["b_l"], (G,), 0.02)
+        if wl.near_tie:
+            rng = _rng(s, layer, 0, TID["near_tie"])
+            for c0_ in range(0, G, 4):
+                for j in range(c0_, min(c0_ + 4, G)):
+                    Wv[j], Wr[j], Wl[j], bl[j] = Wv[c0_], Wr[c0_], Wl[c0_], bl[c0_]
+                    off = 0.0 if c0_ == 0 else float(rng.uniform(0.0, 1e-3))
+                    bv[j] = np.float32(bv[c0_] + np.float32(off))
+        out["W_v"][layer] = _store(Wv, wl.dtype)
+        out["b_v"][layer] = bv
+        out["W_role"][layer] = _store(Wr, wl.dtype)
+        out["W_l"][layer] = _store(Wl, wl.dtype)
+        out["b_l"][layer] = bl
     return out
 
 

@@ -43,13 +43,23 @@ def make_rolesub(wl):
                    wl.n_query_array())
 
 
-def run_gpu(wl, inp, rs=None):
-    """compress + attend on the GPU; returns numpy packed, idx, o and the status."""
+def run_gpu(wl, inp, rs=None, add=None):
+    """compress + attend on the GPU; returns numpy packed, idx, o and the status.
+
+    add: weights of the additive routing score (synth.gen_additive_weights);
+    when given, compress runs rolesub_compress_additive instead.
+    """
     import torch
     rs = rs or make_rolesub(wl)
     dev = {k: to_torch(v, wl.dtype) for k, v in inp.items()}
-    packed, idx = rs.compress(dev["h"], dev["v"], dev["R"], dev["W_re"], dev["b_re"], dev["W1"],
-                              dev["b1"], dev["W2"], dev["b2"], wl.alpha_role, wl.alpha_lang)
+    if add is None:
+        packed, idx = rs.compress(dev["h"], dev["v"], dev["R"], dev["W_re"], dev["b_re"], dev["W1"],
+                                  dev["b1"], dev["W2"], dev["b2"], wl.alpha_role, wl.alpha_lang)
+    else:
+        da = {k: to_torch(v, wl.dtype) for k, v in add.items()}
+        packed, idx = rs.compress_additive(dev["h"], dev["v"], dev["R"], dev["W_re"], dev["b_re"], da["W_v"],
+                                           da["b_v"], da["W_role"], da["W_l"], da["b_l"], wl.alpha_role,
+                                           wl.alpha_lang)
     o = rs.attend(dev["q"], dev["K"], packed, idx, dev["R"])
     torch.cuda.synchronize()
     status = rs.device_status()
@@ -58,8 +68,11 @@ def run_gpu(wl, inp, rs=None):
 
 
 
-def check_layer_episode(wl, inp, gpu, layer, e, report=None):
+def check_layer_episode(wl, inp, gpu, layer, e, report=None, add=None):
     """Oracle compress + attend of one (layer, episode); compares with the GPU.
+
+    add: the additive router's weights when the GPU ran that router; the
+    oracle then routes with compress_layer_linear.
 
     Returns a dict of statistics; raises AssertionError on any violation.
     """
@@ -82,7 +95,14 @@ def check_layer_episode(wl, inp, gpu, layer, e, report=None):
     args = (R, W("W_re"), inp["b_re"][layer].astype(np.float64), W("W1"),
             inp["b1"][layer].astype(np.float64), W("W2"), inp["b2"][layer].astype(np.float64),
             wl.alpha_role, wl.alpha_lang)
-    ref = oracle.compress_layer(spec, h, v, *args)
+    if add is None:
+        ref = oracle.compress_layer(spec, h, v, *args)
+    else:
+        A = lambda name: synth.widen(add[name][layer], wl.dtype)
+        ref = oracle.compress_layer_linear(
+            spec, h, v, R, W("W_re"), inp["b_re"][layer].astype(np.float64), A("W_v"),
+            add["b_v"][layer].astype(np.float64), A("W_role"), A("W_l"), add["b_l"][layer].astype(np.float64),
+            wl.alpha_role, wl.alpha_lang, want_z=False)
 
     # ---- group indices -------------------------------------------------
     gidx = gpu["idx"][layer]

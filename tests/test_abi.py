@@ -167,3 +167,31 @@ def test_calls_reject_bad_arguments_before_any_launch(rsm):
     at2 = [ctypes.byref(s2), p2.host_ptr, fake, fake, 80 * 16, 80, 40, fake, 80 * 16, 80, 40, fake, fake,
            fake, 0.0, fake, fake, 1 << 30, None]
     assert L.rolesub_attend(*at2) == 2
+
+
+def test_additive_compress_rejects_bad_arguments_before_any_launch(rsm):
+    shape = rsm.make_shape(1, 2, 8, 4, 3, 8, "f32")
+    plan = rsm.Plan(shape, [[3, 2, 0, 0]], [[2, 4, 4, 4]], [1])
+    L = rsm.lib()
+    fake = 1 << 20    # never dereferenced: validation fails first
+    # shape, plan, plan_dev, h v R W_re b_re W_v b_v W_role W_l b_l, alphas, packed idx ws ws_bytes stream
+    args = [ctypes.byref(shape), plan.host_ptr, fake] + [fake] * 10 + [0.1, 0.1, fake, fake, fake, 1 << 30, None]
+    for pos in range(3, 13):          # every weight or input pointer null
+        a = list(args)
+        a[pos] = None
+        assert L.rolesub_compress_additive(*a) == 1, pos
+    a = list(args)
+    a[9] = fake + 4                   # b_v not 16-byte aligned
+    assert L.rolesub_compress_additive(*a) == 1
+    a = list(args)
+    a[13] = float("inf")
+    assert L.rolesub_compress_additive(*a) == 1
+    a = list(args)
+    a[18] = 16                        # workspace too small
+    assert L.rolesub_compress_additive(*a) == 1
+    # more role components than the fallback's shared-memory scratch holds
+    big = rsm.make_shape(1, 2, 8, 4, 5000, 8, "f32")
+    pb = rsm.Plan(big, [[3, 2, 0, 0]], [[2, 4, 4, 4]], [1])
+    a = list(args)
+    a[0], a[1] = ctypes.byref(big), pb.host_ptr
+    assert L.rolesub_compress_additive(*a) == 2
