@@ -93,6 +93,25 @@ def compress_bytes(wl):
     return per_layer * wl.L
 
 
+def compress_additive_bytes(wl, C):
+    """Algorithmic bytes of one rolesub_compress_additive over the workload.
+
+    As compress_bytes, with the additive router's weights (W_re [C][d],
+    W_v and W_l [S][d], W_role [S][C], fp32 biases) instead of the
+    concatenation router's.
+    """
+    b = 2 if wl.dtype == "bf16" else 4
+    d, H, ds, G = wl.d, wl.H, wl.dh // wl.G, wl.G
+    per_layer = H * wl.dh * wl.dh * b + (C * d + 2 * G * d + G * C) * b + 4 * (C + 2 * G)
+    for ep in wl.episodes:
+        for kind, (n, k) in enumerate(zip(ep.n_tok(), ep.k(G))):
+            if 0 < k < G or kind == 1:
+                per_layer += n * d * b
+            if k > 0:
+                per_layer += n * d * b + n * k * H * ds * b + n * k
+    return per_layer * wl.L
+
+
 def attend_flops(wl):
     d, H, ds = wl.d, wl.H, wl.dh // wl.G
     f = 0
@@ -385,6 +404,39 @@ def run_ours(args):
     qtok = wl.q_rows * wl.L
     ms_per_step, value = weak_scaling(sum(t_step), args.steps, qtok, ws)
 
+    # ---- the additive routing score (Sec. 3.4) in place of the concatenation
+    # router, same cache, C = 6 role components; timed on its own, after the
+    # step --------------------------------------------------------------------
+    import dataclasses
+    C_ADD = 6
+    wl_add = dataclasses.replace(wl, C=C_ADD)
+    rs_add = rolesub.RoleSub(wl.L, wl.H, wl.dh, wl.G, C_ADD, wl.F, wl.dtype, wl.n_tok_array(), wl.k_array(),
+                             wl.n_query_array(), device=dev)
+    add = {k: to_dev(v) for k, v in synth.gen_additive_weights(wl_add).items()}
+    W_re_add = d["W_re"][:, :C_ADD].contiguous()
+    b_re_add = d["b_re"][:, :C_ADD].contiguous()
+
+    def compress_additive():
+        rs_add.compress_additive(d["h"], d["v"], d["R"], W_re_add, b_re_add, add["W_v"], add["b_v"],
+                                 add["W_role"], add["W_l"], add["b_l"], wl.alpha_role, wl.alpha_lang,
+                                 packed=packed, idx=idx)
+
+    for _ in range(3):
+        compress_additive()
+    torch.cuda.synchronize()
+    ev_add = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(args.steps)]
+    for i in range(args.steps):
+        if flush_buf is not None:
+            flush_buf.fill_(i & 0xFF)
+        ev_add[i][0].record(stream)
+        compress_additive()
+        ev_add[i][1].record(stream)
+    torch.cuda.synchronize()
+    code, _ = rs_add.device_status()
+    assert code == 0, f"device status {code}"
+    add_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_add)
+
     # ---- end to end through the public API from pinned host buffers --------
     act = ("h", "v", "K", "q")
     host = {}
@@ -436,6 +488,9 @@ def run_ours(args):
             "tensor_tflops": attend_flops(wl) / (att_ms / 1e3) / 1e12}
     comp = {"ms": comp_ms, "algorithmic_bytes": cb, "GB/s": cb / (comp_ms / 1e3) / 1e9,
             "frac": cb / (comp_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
+    cab = compress_additive_bytes(wl, C_ADD)
+    comp_add = {"ms": add_ms, "role_dim": C_ADD, "algorithmic_bytes": cab, "GB/s": cab / (add_ms / 1e3) / 1e9,
+                "frac": cab / (add_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
 
     clocks = clk.summary()
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
@@ -446,7 +501,7 @@ def run_ours(args):
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "ms_per_step": e2e_ms},
             "gpu_launches": launches,
-            "roofline": roof, "compress": comp,
+            "roofline": roof, "compress": comp, "compress_additive": comp_add,
             "clocks": {"sm_mhz": clocks["sm_mhz"], "sm_max_mhz": clocks["sm_max_mhz"],
                        "reasons": clocks["reasons"], "samples": clocks["samples"]}}
     if ws == 1 and rank == 0 and not args.no_cpu_baseline:

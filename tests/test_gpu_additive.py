@@ -90,3 +90,14 @@ def test_additive_rejects_oversized_role_dim():
     with pytest.raises(R.RoleSubError) as ei:
         rs.compress_additive(z, z, z, z, z, z, z, z, z, z)
     assert ei.value.code == 2
+
+
+@pytest.mark.slow
+def test_additive_c4_full_size_sampled():
+    """The batched ragged workload at full size (64 episodes, 32 layers) in
+    the launch configuration the benchmark times, checked on sampled
+    (layer, episode) pairs."""
+    wl = dataclasses.replace(synth.c4(), C=6)
+    sizes = [ep.n_cache for ep in wl.episodes]
+    e_big, e_small = int(np.argmax(sizes)), int(np.argmin(sizes))
+    _run(wl, [(0, e_big), (31, e_small), (17, 5), (5, 40)])
