@@ -32,7 +32,7 @@
 // O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into the unit's Y buffer, output
 // stores.
 //
-// Warp roles (512 threads), all hand-offs through mbarriers. Warp w runs on
+// Warp roles (544 threads), all hand-offs through mbarriers. Warp w runs on
 // sub-partition w % 4.
 //   warps 0-3   softmax, one per TMEM lane quadrant
 //   warps 4-5, 12-13  value gather, one kv row per thread: warps 4-5 the
@@ -40,7 +40,9 @@
 //   warp 6      issues S = Q K^T, chunk by chunk
 //   warp 14     issues Y += P Z, chunk by chunk
 //   warp 15     issues O = Y R_h^T, unit by unit
-//   warp 7      TMA producer: K (3-slot ring), Q (2 slots), R_h
+//   warp 7      TMA producer of K (3-slot ring), chunk by chunk
+//   warp 16     TMA producer of Q (2 slots) and R_h, unit by unit (apart
+//               from the K producer, so that neither's waits hold up the other)
 //   warps 8-11  unit tail, one per lane quadrant, overlapping the next
 //               unit's chunks (Y is double buffered in TMEM)
 // S and P have three buffers and Z four slots: a chunk's S product waits for
@@ -75,7 +77,7 @@ namespace {
 using namespace sm100;
 typedef __nv_bfloat16 bf16;
 
-constexpr int kThreads = 512;
+constexpr int kThreads = 544;
 constexpr int kChunk = 64;   // cache tokens per chunk
 constexpr int kQRows = 64;   // query rows per unit
 constexpr int kDh = 128;
@@ -264,14 +266,13 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
     const uint32_t tmem = tmem_slot;
 
     if (warp == 7) {
-        // ================= TMA producer =================================
+        // ================= TMA producer: keys =============================
         if (lane == 0) {
             prefetch_tmap(&tm_q);
             prefetch_tmap(&tm_k);
             prefetch_tmap(&tm_r);
             ChunkIt it = first;
-            uint32_t n = 0, g = 0;
-            int run = -1, pl = -1, ph = -1;
+            uint32_t g = 0;
             auto load_k = [&](const Unit &t, int c) -> bool {
                 const uint32_t ks = g % kKSlots;
                 if (g >= kKSlots && !mbar_wait(B(B_KE + ks), ((g / kKSlots) - 1) & 1, status, &abort_flag, 41))
@@ -283,15 +284,21 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 ++g;
                 return true;
             };
-            bool ok = true;
-            while (ok && it.k < nu) {
+            while (it.k < nu) {
+                if (!load_k(it.t, it.c)) break;
+                it_next(sp, it, nu);
+            }
+        }
+    } else if (warp == 16) {
+        // ================= TMA producer: Q and R_h ======================
+        // Q of unit n waits for its slot (unit n - 2's last S product); R_h
+        // of a new (layer, head) for the previous run's last output product
+        if (lane == 0) {
+            ChunkIt it = first;
+            uint32_t n = 0;
+            int run = -1, pl = -1, ph = -1;
+            while (it.k < nu) {
                 const Unit t = it.t;
-                // keys that fit the ring first (they only wait for older products),
-                // then Q (its slot frees when unit n-2 has its output), then R_h of
-                // a new (layer, head) once the previous run is done, then the rest
-                const int head = min(t.nch, kKSlots);
-                for (int c = 0; c < head && ok; ++c) ok = load_k(t, c);
-                if (!ok) break;
                 const uint32_t qs = n & 1;
                 if (n >= 2 && !mbar_wait(B(B_QE + qs), ((n >> 1) - 1) & 1, status, &abort_flag, 40)) break;
                 mbar_expect_tx(B(B_QF + qs), 16384);
@@ -306,7 +313,6 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                     pl = t.l;
                     ph = t.h;
                 }
-                for (int c = head; c < t.nch && ok; ++c) ok = load_k(t, c);
                 next_unit(sp, it, nu);
                 ++n;
             }
