@@ -8,8 +8,9 @@
 //
 // Kernels, in order:
 //   language pool      the concatenation router's pooling kernels
-//   k_lang_term_add    beta_e = alpha_lang (W_l c_e + b_l), a warp per
-//                      (layer, episode, group), fp32
+//   k_lang_term_add4   beta_e = alpha_lang (W_l c_e + b_l), fp32: a block
+//                      per (layer, 4 episodes), S <= 16 (k_lang_term_add, a
+//                      warp per (layer, episode, group), above that)
 //   k_router_add_tc    bf16, S = 16: one CTA per (128-row router tile,
 //                      layer); a single tcgen05 product [W_v ; W_re] h over
 //                      d (N = S + C rounded up to 16, zero rows padding it)
@@ -51,6 +52,57 @@ k_lang_term_add(const T *__restrict__ W_l, const float *__restrict__ b_l, const 
     for (int t = lane; t < d; t += 32) acc = fmaf(to_f(w[t]), c[t], acc);
     acc = warp_sum(acc);
     if (lane == 0) beta[((size_t)l * E + e) * G + s] = alpha_lang * (b_l[(size_t)l * G + s] + acc);
+}
+
+// The same for S <= 16: a block of 256 threads per (layer, 4 episodes);
+// thread t takes columns t, t + 256, ... of the four contexts and all S rows
+// of W_l (each W_l element read once per block), then the block sums.
+constexpr int kTermEp = 4, kTermMaxG = 16;
+
+template <class T>
+__global__ void __launch_bounds__(256)
+k_lang_term_add4(const T *__restrict__ W_l, const float *__restrict__ b_l, const float *__restrict__ ctx, int E,
+                 int d, int G, float alpha_lang, float *__restrict__ beta)
+{
+    __shared__ float part[8][kTermEp * kTermMaxG];
+    const int l = blockIdx.y, e0 = blockIdx.x * kTermEp, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    float acc[kTermEp][kTermMaxG];
+#pragma unroll
+    for (int i = 0; i < kTermEp; ++i)
+#pragma unroll
+        for (int s = 0; s < kTermMaxG; ++s) acc[i][s] = 0.f;
+    const T *w = W_l + (size_t)l * G * d;
+    const float *c = ctx + ((size_t)l * E + e0) * d;
+    for (int t = threadIdx.x; t < d; t += 256) {
+        float cv[kTermEp];
+#pragma unroll
+        for (int i = 0; i < kTermEp; ++i) cv[i] = e0 + i < E ? c[(size_t)i * d + t] : 0.f;
+#pragma unroll
+        for (int s = 0; s < kTermMaxG; ++s) {
+            if (s < G) {
+                const float wv = to_f(w[(size_t)s * d + t]);
+#pragma unroll
+                for (int i = 0; i < kTermEp; ++i) acc[i][s] = fmaf(wv, cv[i], acc[i][s]);
+            }
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < kTermEp; ++i)
+#pragma unroll
+        for (int s = 0; s < kTermMaxG; ++s) {
+            const float v = warp_sum(acc[i][s]);
+            if (lane == 0) part[warp][i * kTermMaxG + s] = v;
+        }
+    __syncthreads();
+    if (threadIdx.x < kTermEp * kTermMaxG) {
+        const int i = threadIdx.x / kTermMaxG, s = threadIdx.x % kTermMaxG;
+        if (s < G && e0 + i < E) {
+            float v = 0.f;
+#pragma unroll
+            for (int q = 0; q < 8; ++q) v += part[q][threadIdx.x];
+            beta[((size_t)l * E + e0 + i) * G + s] = alpha_lang * (b_l[(size_t)l * G + s] + v);
+        }
+    }
 }
 
 // One warp per routed row: the S + C dot products over d, the role softmax
@@ -318,8 +370,12 @@ cudaError_t launch_additive_t(const CompressArgs &a, const AdditiveWeights &w)
     if (M == 0) return cudaSuccess;
     cudaError_t err = launch_lang_pool(a);
     if (err != cudaSuccess) return err;
-    k_lang_term_add<T><<<dim3((unsigned)((E * G + 7) / 8), L), 256, 0, a.stream>>>(
-        (const T *)w.W_l, w.b_l, a.ws.lang_ctx, E, d, G, a.alpha_lang, a.ws.lang_bias);
+    if (G <= kTermMaxG)
+        k_lang_term_add4<T><<<dim3((unsigned)((E + kTermEp - 1) / kTermEp), L), 256, 0, a.stream>>>(
+            (const T *)w.W_l, w.b_l, a.ws.lang_ctx, E, d, G, a.alpha_lang, a.ws.lang_bias);
+    else
+        k_lang_term_add<T><<<dim3((unsigned)((E * G + 7) / 8), L), 256, 0, a.stream>>>(
+            (const T *)w.W_l, w.b_l, a.ws.lang_ctx, E, d, G, a.alpha_lang, a.ws.lang_bias);
     count_launches(1);
     if ((err = cudaGetLastError()) != cudaSuccess) return err;
     const PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev,
