@@ -18,6 +18,15 @@ Parity status of each function (what pins it, in tests/test_oracle_pins.py):
                      count against the paper's 4.20M routing heads
   topk            -- brute-force subset enumeration, hand-built near-ties
   rotate          -- permutation matrices, norm preservation
+  budget_shares / budget_allocate -- Sec. 3.5 allocator (reading: rank-linear
+                     weights, water-filled at S, largest remainders): hand-
+                     computed cases, the budget and bound constraints, an
+                     independent bisection water-fill, brute-force nearest
+                     integer vector on tiny cases
+  route_layer_budget / pack_layer_budget / attend_layer_budget -- per-token
+                     K_i: counts from the allocator over pi = u . a (scipy
+                     softmax), brute-force top-K_i, equal counts == the
+                     fixed-k C path, every mask == dense R M R^T v attention
   compress/attend -- all-kept == dense attention (1e-10), none-kept == 0,
                      every mask on tiny inputs == dense attention over
                      R M R^T v, complement linearity, R = I textbook case,
@@ -73,6 +82,14 @@ def lib():
             L.oracle_route_episode_linear.argtypes = (
                 [ctypes.c_int] * 3 + [_ip, _ip, _llp] + [_dp] * 8 + [ctypes.c_double] * 2 + [_ubp, _dp, _dp])
             L.oracle_route_episode_linear.restype = ctypes.c_int
+            L.oracle_budget_shares.argtypes = [ctypes.c_int, ctypes.c_longlong, ctypes.c_int, _ip]
+            L.oracle_budget_shares.restype = ctypes.c_int
+            L.oracle_budget_allocate.argtypes = [ctypes.c_int, ctypes.c_longlong, ctypes.c_int, _dp, _ip]
+            L.oracle_budget_allocate.restype = ctypes.c_int
+            L.oracle_route_episode_budget.argtypes = (
+                [ctypes.c_int] * 3 + [_ip, _ip, _llp] + [_dp] * 9 + [ctypes.c_double] * 2
+                + [_ip, _ubp, _ip, _dp, _dp, _dp])
+            L.oracle_route_episode_budget.restype = ctypes.c_int
             L.oracle_topk.argtypes = [ctypes.c_int, ctypes.c_int, _dp, _ubp, _dp]
             L.oracle_topk.restype = None
             L.oracle_rotate.argtypes = [ctypes.c_int, _dp, _dp, _dp]
@@ -351,4 +368,164 @@ def attend_layer(spec: Spec, q, K, packed, idx, R, scale=0.0, episodes=None, hea
         if rc != 0:
             raise ValueError("oracle_attend_episode: bad arguments or indices")
         o[q0:q1, :] = np.where(np.isin(np.arange(s.d) // s.dh, np.arange(h0, h1))[None, :], oe, o[q0:q1])
+    return o
+
+
+# ---------------------------------------------------------------------------
+# Per-token budgets (Sec. 3.5)
+# ---------------------------------------------------------------------------
+
+def budget_shares(n, B, S):
+    """Counts by priority rank (rank 0 = highest) of the allocator reading."""
+    out = np.zeros(max(n, 1), np.int32)
+    if lib().oracle_budget_shares(int(n), int(B), int(S), out.ctypes.data_as(_ip)) != 0:
+        raise ValueError("oracle_budget_shares: bad arguments")
+    return out[:n]
+
+
+def budget_allocate(pri, B, S):
+    """Per-token counts for priorities pri (ties: lower index ranks higher)."""
+    pri, pp = _d(np.asarray(pri, np.float64).reshape(-1))
+    n = pri.size
+    out = np.zeros(max(n, 1), np.int32)
+    if lib().oracle_budget_allocate(n, int(B), int(S), pp if n else None, out.ctypes.data_as(_ip)) != 0:
+        raise ValueError("oracle_budget_allocate: bad arguments")
+    return out[:n]
+
+
+def budget_idx_offsets(spec: Spec, ktok_layer):
+    """Where each routed token's indices start: per segment, idx_off + the
+    prefix sum of the counts of the tokens before it (Sec. 3.5 packing)."""
+    lay = spec.lay
+    nt = spec.n_tok.reshape(-1)
+    out = np.zeros(int(spec.ep_row[-1]), np.int64)
+    for sgi in range(nt.size):
+        r0, n = int(lay["row_off"][sgi]), int(nt[sgi])
+        if n:
+            kk = np.asarray(ktok_layer[r0:r0 + n], np.int64)
+            out[r0:r0 + n] = lay["idx_off"][sgi] + np.concatenate([[0], np.cumsum(kk)[:-1]])
+    return out
+
+
+def route_layer_budget(spec: Spec, h, W_re, b_re, W_v, b_v, W_role, W_l, b_l, u, alpha_role, alpha_lang,
+                       episodes=None, k_force=None):
+    """Additive-router scores, priorities pi = u . a and per-token budgets for
+    every (listed) episode of one layer; returns idx [idx_bytes] uint8,
+    ktok [rows] int32, gamma [rows][G], pri [rows], margin [rows]."""
+    s = spec
+    lay = s.lay
+    rows = int(s.ep_row[-1])
+    idx = np.zeros(max(lay["idx_bytes"], 1), np.uint8)
+    ktok = np.zeros(max(rows, 1), np.int32)
+    gamma = np.full((max(rows, 1), s.G), np.nan)
+    pri = np.full(max(rows, 1), np.nan)
+    margin = np.full(max(rows, 1), np.nan)
+    Wre, Wrep = _d(W_re)
+    bre, brep = _d(b_re)
+    Wv, Wvp = _d(W_v)
+    bv, bvp = _d(b_v)
+    Wr, Wrp = _d(W_role)
+    Wl, Wlp = _d(W_l)
+    bl, blp = _d(b_l)
+    uu, up = _d(u)
+    kf = None if k_force is None else np.ascontiguousarray(k_force, np.int32)
+    for e in (range(s.E) if episodes is None else episodes):
+        r0, r1 = int(s.ep_row[e]), int(s.ep_row[e + 1])
+        n = max(r1 - r0, 1)
+        he, hp = _d(h[r0:r1] if r1 > r0 else np.zeros((1, s.d)))
+        nt, ntp = _i(s.n_tok[e])
+        kk, kp = _i(s.k[e])
+        io, iop = _ll(lay["idx_off"][4 * e:4 * e + 4])
+        kt = np.zeros(n, np.int32)
+        g_e = np.full((n, s.G), np.nan)
+        p_e = np.full(n, np.nan)
+        m_e = np.full(n, np.nan)
+        kfe = None if kf is None else np.ascontiguousarray(
+            kf[r0:r1] if r1 > r0 else np.zeros(1, np.int32), np.int32)
+        rc = lib().oracle_route_episode_budget(
+            s.d, s.G, s.C, ntp, kp, iop, hp, Wrep, brep, Wvp, bvp, Wrp, Wlp, blp, up, float(alpha_role),
+            float(alpha_lang), None if kfe is None else kfe.ctypes.data_as(_ip), _u8(idx),
+            kt.ctypes.data_as(_ip), g_e.ctypes.data_as(_dp), p_e.ctypes.data_as(_dp), m_e.ctypes.data_as(_dp))
+        if rc != 0:
+            raise ValueError("oracle_route_episode_budget: bad arguments or forced counts")
+        ktok[r0:r1] = kt[:r1 - r0]
+        gamma[r0:r1] = g_e[:r1 - r0]
+        pri[r0:r1] = p_e[:r1 - r0]
+        margin[r0:r1] = m_e[:r1 - r0]
+    return {"idx": idx[:lay["idx_bytes"]], "ktok": ktok[:rows], "gamma": gamma[:rows], "pri": pri[:rows],
+            "margin": margin[:rows]}
+
+
+def pack_layer_budget(spec: Spec, v, R, idx, ktok, episodes=None):
+    """Sec. 3.2 with per-token counts: z = R_h^T v_{i,h}; segment of n tokens
+    holds [H][sum_i K_i][d_s] values, token i's kept groups at the prefix
+    sum of the counts before it, in its index order. Returns packed
+    [packed_elems] float64 (unlisted episodes stay zero)."""
+    s = spec
+    lay = s.lay
+    ds = s.dh // s.G
+    packed = np.zeros(max(lay["packed_elems"], 1))
+    nt = s.n_tok.reshape(-1)
+    R = np.asarray(R, np.float64)
+    eps = range(s.E) if episodes is None else episodes
+    for e in eps:
+        for m in range(4):
+            sgi = 4 * e + m
+            n, r0 = int(nt[sgi]), int(lay["row_off"][sgi])
+            if n == 0:
+                continue
+            kk = np.asarray(ktok[r0:r0 + n], np.int64)
+            tot = int(kk.sum())
+            pref = np.concatenate([[0], np.cumsum(kk)[:-1]])
+            io, po = int(lay["idx_off"][sgi]), int(lay["packed_off"][sgi])
+            for hh in range(s.H):
+                z = np.asarray(v[r0:r0 + n, hh * s.dh:(hh + 1) * s.dh], np.float64) @ R[hh]   # rows: z = R^T v
+                for i in range(n):
+                    for j in range(int(kk[i])):
+                        g = int(idx[io + pref[i] + j])
+                        dst = po + (hh * tot + pref[i] + j) * ds
+                        packed[dst:dst + ds] = z[i, g * ds:(g + 1) * ds]
+    return packed[:lay["packed_elems"]]
+
+
+def attend_layer_budget(spec: Spec, q, K, packed, idx, ktok, R, scale=0.0, episodes=None):
+    """Attention over a cache packed with per-token counts (Sec. 3):
+    p = softmax_j(q . k_j * scale) over the episode's cache tokens,
+    y = sum_j p_j M_j z_j (zeros outside the kept groups), o = R_h y.
+    Returns o [q_rows][d] float64."""
+    s = spec
+    lay = s.lay
+    ds = s.dh // s.G
+    sc = scale if scale > 0 else 1.0 / np.sqrt(s.dh)
+    o = np.zeros((int(s.ep_q[-1]), s.d))
+    nt = s.n_tok.reshape(-1)
+    R = np.asarray(R, np.float64)
+    for e in (range(s.E) if episodes is None else episodes):
+        r0, r1 = int(s.ep_row[e]), int(s.ep_row[e + 1])
+        q0, q1 = int(s.ep_q[e]), int(s.ep_q[e + 1])
+        if q1 == q0 or r1 == r0:
+            continue
+        for hh in range(s.H):
+            ztil = np.zeros((r1 - r0, s.dh))
+            for m in range(4):
+                sgi = 4 * e + m
+                n, rs_ = int(nt[sgi]), int(lay["row_off"][sgi])
+                if n == 0:
+                    continue
+                kk = np.asarray(ktok[rs_:rs_ + n], np.int64)
+                tot = int(kk.sum())
+                pref = np.concatenate([[0], np.cumsum(kk)[:-1]])
+                io, po = int(lay["idx_off"][sgi]), int(lay["packed_off"][sgi])
+                for i in range(n):
+                    for j in range(int(kk[i])):
+                        g = int(idx[io + pref[i] + j])
+                        src = po + (hh * tot + pref[i] + j) * ds
+                        ztil[rs_ - r0 + i, g * ds:(g + 1) * ds] = packed[src:src + ds]
+            qh = np.asarray(q[q0:q1, hh * s.dh:(hh + 1) * s.dh], np.float64)
+            kh = np.asarray(K[r0:r1, hh * s.dh:(hh + 1) * s.dh], np.float64)
+            sco = qh @ kh.T * sc
+            sco -= sco.max(axis=1, keepdims=True)
+            p = np.exp(sco)
+            p /= p.sum(axis=1, keepdims=True)
+            o[q0:q1, hh * s.dh:(hh + 1) * s.dh] = (p @ ztil) @ R[hh].T
     return o

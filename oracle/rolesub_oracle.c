@@ -20,6 +20,11 @@
  *             group index first). oracle_router_score_linear is the
  *             additive form as printed (linear f_v and f_lang heads, W_role
  *             a, each term weighted as in the equation).
+ *   Sec. 3.5  per-token budgets: within a token type, K_i of the S groups
+ *             with sum_i K_i = K_m |I_m|, more for higher role-derived
+ *             priority (oracle_budget_*: the allocator as read here);
+ *             packed with each token's groups at the prefix sum of the
+ *             counts before it.
  *   Attention (Sec. 3, keys and queries unchanged; values routed):
  *             s_j = q . k_j * scale, p = softmax_j(s) over every cache token
  *             of the episode (non-causal), o = sum_j p_j v~_j, evaluated as
@@ -423,4 +428,183 @@ int oracle_attend_episode(int H, int dh, int G, const int *n_tok, const int *k,
     free(y);
     free(ztil);
     return 0;
+}
+
+/*
+ * Role-driven budget allocation, Sec. 3.5 (the allocator B^(l)). The paper
+ * fixes its constraints -- 0 <= K_i <= S and sum_i K_i = B_m = K_m |I_m| for
+ * the tokens of one type -- and that tokens of higher role-derived priority
+ * get more value groups; it gives no formula. Reading used here:
+ *   - rank the n tokens by priority (higher first, ties: lower token index);
+ *   - rank r (0-based) has weight n - r;
+ *   - real shares x_r = min(S, lambda (n - r)), lambda chosen so that
+ *     sum_r x_r = B (the best ranks saturate at S first);
+ *   - K is x rounded by largest remainders: floor(x_r), plus one for the
+ *     B - sum floor(x_r) ranks with the largest fractional parts (ties: the
+ *     better rank).
+ * Once the ranks are fixed everything is integer arithmetic: with c ranks
+ * saturated, x_r = (B - cS)(n - r) / W_c for r >= c, W_c = sum_{r>=c}(n - r).
+ * K_by_rank[r] receives the count of rank r. Returns 0, or -1 on bad
+ * arguments (B outside [0, nS]).
+ */
+int oracle_budget_shares(int n, long long B, int S, int *K_by_rank)
+{
+    if (n < 0 || S < 0 || B < 0 || B > (long long)n * S) return -1;
+    if (n == 0) return 0;
+    /* number of saturated ranks: the first c whose largest unsaturated share
+     * (rank c) does not exceed S */
+    int c = 0;
+    for (; c < n; ++c) {
+        long long rest = B - (long long)c * S;
+        long long W = (long long)(n - c) * (n - c + 1) / 2;
+        if (rest * (long long)(n - c) <= (long long)S * W) break;
+    }
+    for (int r = 0; r < c; ++r) K_by_rank[r] = S;
+    if (c == n) return 0;
+    long long rest = B - (long long)c * S;
+    long long W = (long long)(n - c) * (n - c + 1) / 2;
+    long long assigned = 0;
+    long long *rem = (long long *)malloc(sizeof(long long) * (size_t)n);
+    for (int r = c; r < n; ++r) {
+        long long num = rest * (long long)(n - r);
+        K_by_rank[r] = (int)(num / W);
+        rem[r] = num % W;
+        assigned += K_by_rank[r];
+    }
+    /* the left-over groups, one each, to the largest remainders */
+    long long left = rest - assigned;
+    for (long long t = 0; t < left; ++t) {
+        int best = -1;
+        for (int r = c; r < n; ++r)
+            if (rem[r] >= 0 && (best < 0 || rem[r] > rem[best])) best = r;
+        K_by_rank[best] += 1;
+        rem[best] = -1; /* taken */
+    }
+    free(rem);
+    return 0;
+}
+
+/* The allocation of one token type: ranks the n priorities (higher first,
+ * ties: lower index) and gives token i the count of its rank.
+ * Returns 0, or -1 on bad arguments. */
+int oracle_budget_allocate(int n, long long B, int S, const double *pri, int *K)
+{
+    if (n < 0) return -1;
+    if (n == 0) return 0;
+    int *byrank = (int *)malloc(sizeof(int) * (size_t)n);
+    if (oracle_budget_shares(n, B, S, byrank) != 0) {
+        free(byrank);
+        return -1;
+    }
+    for (int i = 0; i < n; ++i) {
+        int rank = 0;
+        for (int j = 0; j < n; ++j)
+            if (pri[j] > pri[i] || (pri[j] == pri[i] && j < i)) ++rank;
+        K[i] = byrank[rank];
+    }
+    free(byrank);
+    return 0;
+}
+
+/*
+ * Routing of one episode of one layer with per-token budgets (Sec. 3.4 and
+ * Sec. 3.5): the additive score of oracle_router_score_linear, the latent
+ * role a_i of Eq. (latentrole) and the priority pi_i = u . a_i. For a segment
+ * of n tokens with target K_m (k[m]):
+ *   0 < K_m < G  K_i from oracle_budget_allocate(pi, B = K_m n), unless
+ *                k_force_ep gives them ([n_cache], summing to B); the
+ *                K_i largest scores are kept (oracle_topk) and written at
+ *                idx_off[m] + sum_{j<i} K_j;
+ *   K_m = G      every token keeps every group (indices 0..G-1);
+ *   K_m = 0      nothing is kept.
+ * Outputs: idx_layer at the segment offsets; ktok_ep [n_cache] = K_i; and
+ * optionally gamma_ep [n_cache][G] and pri_ep [n_cache] (NaN where the
+ * router does not run) and margin_ep [n_cache] (top-K_i margin).
+ * Returns 0, or -1 on bad arguments or forced counts that break the budget.
+ */
+int oracle_route_episode_budget(int d, int G, int C, const int *n_tok, const int *k,
+                                const long long *idx_off, const double *h_ep,
+                                const double *W_re, const double *b_re,
+                                const double *W_v, const double *b_v, const double *W_role,
+                                const double *W_l, const double *b_l, const double *u,
+                                double alpha_role, double alpha_lang, const int *k_force_ep,
+                                unsigned char *idx_layer, int *ktok_ep, double *gamma_ep,
+                                double *pri_ep, double *margin_ep)
+{
+    if (d <= 0 || G <= 0 || G > 64 || C < 1) return -1;
+    int row0[OR_KINDS];
+    int nc = 0;
+    for (int m = 0; m < OR_KINDS; ++m) {
+        if (n_tok[m] < 0 || k[m] < 0 || k[m] > G) return -1;
+        row0[m] = nc;
+        nc += n_tok[m];
+    }
+    double *c = (double *)malloc(sizeof(double) * (size_t)d);
+    oracle_lang_pool(d, n_tok[1], h_ep + (size_t)row0[1] * d, c);
+    double *a = (double *)malloc(sizeof(double) * (size_t)C);
+    double *gam = (double *)malloc(sizeof(double) * (size_t)(nc > 0 ? nc : 1) * G);
+    double *pri = (double *)malloc(sizeof(double) * (size_t)(nc > 0 ? nc : 1));
+    int rc = 0;
+    for (int m = 0; m < OR_KINDS && rc == 0; ++m) {
+        int n = n_tok[m], km = k[m];
+        for (int i = 0; i < n; ++i) {
+            int r = row0[m] + i;
+            pri[r] = NAN;
+            for (int g = 0; g < G; ++g) gam[(size_t)r * G + g] = NAN;
+            if (margin_ep) margin_ep[r] = INFINITY;
+        }
+        if (km == G) {
+            for (int i = 0; i < n; ++i) {
+                ktok_ep[row0[m] + i] = G;
+                for (int g = 0; g < G; ++g) idx_layer[idx_off[m] + (long long)i * G + g] = (unsigned char)g;
+            }
+            continue;
+        }
+        if (km == 0) {
+            for (int i = 0; i < n; ++i) ktok_ep[row0[m] + i] = 0;
+            continue;
+        }
+        for (int i = 0; i < n; ++i) {
+            int r = row0[m] + i;
+            const double *h = h_ep + (size_t)r * d;
+            oracle_role(d, C, W_re, b_re, h, a);
+            double p = 0.0;
+            for (int t = 0; t < C; ++t) p += u[t] * a[t];
+            pri[r] = p;
+            oracle_router_score_linear(d, C, G, W_v, b_v, W_role, W_l, b_l, h, a, c, alpha_role,
+                                       alpha_lang, gam + (size_t)r * G);
+        }
+        long long B = (long long)km * n;
+        if (k_force_ep) {
+            long long s = 0;
+            for (int i = 0; i < n; ++i) {
+                int kk = k_force_ep[row0[m] + i];
+                if (kk < 0 || kk > G) rc = -1;
+                ktok_ep[row0[m] + i] = kk;
+                s += kk;
+            }
+            if (s != B) rc = -1;
+            if (rc != 0) break;
+        } else if (oracle_budget_allocate(n, B, G, pri + row0[m], ktok_ep + row0[m]) != 0) {
+            rc = -1;
+            break;
+        }
+        long long off = idx_off[m];
+        for (int i = 0; i < n; ++i) {
+            int r = row0[m] + i, kk = ktok_ep[r];
+            double mg;
+            oracle_topk(G, kk, gam + (size_t)r * G, idx_layer + off, &mg);
+            if (margin_ep) margin_ep[r] = mg;
+            off += kk;
+        }
+    }
+    if (gamma_ep)
+        for (size_t t = 0; t < (size_t)nc * G; ++t) gamma_ep[t] = gam[t];
+    if (pri_ep)
+        for (int t = 0; t < nc; ++t) pri_ep[t] = pri[t];
+    free(c);
+    free(a);
+    free(gam);
+    free(pri);
+    return rc;
 }

@@ -584,3 +584,190 @@ def test_additive_router_compress_keeps_best_subset_and_packs_rotated_groups(ora
             base = lay["packed_off"][m] + ((hh * n + i) * kk) * ds
             want = np.concatenate([z[g * ds:(g + 1) * ds] for g in sel])
             assert np.max(np.abs(out["packed"][base:base + kk * ds] - want)) < 1e-12
+
+
+# ---------------------------------------------------------------------------
+# Per-token budgets (Sec. 3.5). The allocator's formula is this build's
+# reading (rank-linear weights, water-filled at S, largest remainders); the
+# paper fixes its constraints, pinned here with independent computations.
+# ---------------------------------------------------------------------------
+
+def _waterfill(n, B, S):
+    """Real shares x_r = min(S, lam * (n - r)) with sum x = B, by bisection
+    on lam (independent of the oracle's integer closed form)."""
+    w = np.arange(n, 0, -1, dtype=np.float64)
+    if B == n * S:
+        return np.full(n, float(S))
+    lo, hi = 0.0, float(S)
+    for _ in range(200):
+        lam = 0.5 * (lo + hi)
+        if np.minimum(S, lam * w).sum() < B:
+            lo = lam
+        else:
+            hi = lam
+    return np.minimum(S, hi * w)
+
+
+@pytest.mark.parametrize("n,B,S,want", [
+    (4, 8, 16, [3, 2, 2, 1]),      # x = 3.2 2.4 1.6 0.8 -> floors 3 2 1 0, two left to .8, .6
+    (3, 6, 16, [3, 2, 1]),         # exact shares
+    (2, 7, 4, [4, 3]),             # rank 0 saturates (x would be 4.67 > S)
+    (5, 80, 16, [16] * 5),         # K_m = S: everything kept
+    (5, 0, 16, [0] * 5),           # K_m = 0: nothing kept
+    (1, 9, 16, [9]),               # a single token takes the whole budget
+])
+def test_budget_shares_hand_computed(oracle, n, B, S, want):
+    assert list(oracle.budget_shares(n, B, S)) == want
+
+
+def test_budget_shares_constraints_and_nearest_integers(oracle):
+    rng = np.random.default_rng(40)
+    for _ in range(300):
+        S = int(rng.choice([4, 8, 16]))
+        n = int(rng.integers(1, 70))
+        Km = int(rng.integers(0, S + 1))
+        B = Km * n
+        K = oracle.budget_shares(n, B, S).astype(np.int64)
+        x = _waterfill(n, B, S)
+        assert K.sum() == B and K.min() >= 0 and K.max() <= S          # Sec. 3.5 constraints
+        assert np.all(np.diff(K) <= 0)                                   # better rank, no fewer groups
+        assert np.all(np.abs(K - x) < 1.0 + 1e-9)                        # a rounding of the shares
+        # largest remainders: every rank rounded up has a fractional part no
+        # smaller than every rank rounded down
+        fr = x - np.floor(x + 1e-12)
+        up = K > np.floor(x + 1e-12)
+        if up.any() and (~up).any():
+            assert fr[up].min() >= fr[~up & (fr > 1e-9)].max(initial=0.0) - 1e-9
+
+
+def test_budget_shares_minimise_distance_brute_force(oracle):
+    # the integer vector with the budget's sum and bounds closest to the real
+    # shares (least squares), by enumeration, when that minimiser is unique
+    for S in (2, 3, 4):
+        for n in range(1, 6):
+            for Km in range(S + 1):
+                B = Km * n
+                x = _waterfill(n, B, S)
+                cands = [c for c in itertools.product(range(S + 1), repeat=n) if sum(c) == B]
+                dist = [float(np.sum((np.array(c) - x) ** 2)) for c in cands]
+                best = min(dist)
+                winners = [c for c, dd in zip(cands, dist) if abs(dd - best) < 1e-9]
+                K = tuple(int(v) for v in oracle.budget_shares(n, B, S))
+                if len(winners) == 1:
+                    assert K == winners[0], (S, n, Km, K, winners)
+                else:   # tied fractional parts: the better ranks round up
+                    assert K in winners and K == max(winners), (S, n, Km, K, winners)
+
+
+def test_budget_allocate_follows_priority_ranks(oracle):
+    rng = np.random.default_rng(41)
+    pri = rng.standard_normal(9)
+    K = oracle.budget_allocate(pri, 9 * 5, 16)
+    byrank = oracle.budget_shares(9, 45, 16)
+    order = np.argsort(-pri, kind="stable")
+    assert list(K[order]) == list(byrank)
+    perm = rng.permutation(9)
+    assert list(oracle.budget_allocate(pri[perm], 45, 16)) == list(K[perm])   # token order irrelevant
+    # equal priorities: the lower token index ranks first
+    assert list(oracle.budget_allocate([0.5, 0.5, 0.5, 0.5], 8, 16)) == [3, 2, 2, 1]
+
+
+def _budget_problem(rng, n_tok, k, G=4, H=2, dh=8, C=3):
+    p = rnd_problem(rng, H=H, dh=dh, G=G, C=C, F=4, n_tok=n_tok, k=k, n_q=tuple(3 for _ in n_tok))
+    d = H * dh
+    p["W_v"] = 0.3 * rng.standard_normal((G, d))
+    p["b_v"] = 0.3 * rng.standard_normal(G)
+    p["W_role"] = rng.standard_normal((G, C))
+    p["W_l"] = 0.3 * rng.standard_normal((G, d))
+    p["b_l"] = 0.3 * rng.standard_normal(G)
+    p["u"] = rng.standard_normal(C)
+    return p
+
+
+def _route_budget(oracle, p, k_force=None):
+    spec = oracle.Spec(p["H"], p["dh"], p["G"], p["C"], p["F"], p["n_tok"], p["k"], p["n_q"])
+    out = oracle.route_layer_budget(spec, p["h"], p["W_re"], p["b_re"], p["W_v"], p["b_v"], p["W_role"], p["W_l"],
+                                    p["b_l"], p["u"], 0.1, 0.1, k_force=k_force)
+    return spec, out
+
+
+def test_budget_routing_counts_priorities_and_best_subsets(oracle):
+    rng = np.random.default_rng(42)
+    G = 4
+    p = _budget_problem(rng, n_tok=((7, 4, 0, 0), (3, 2, 2, 0)), k=((2, 1, G, G), (3, 0, 0, G)), G=G)
+    spec, out = _route_budget(oracle, p)
+    lay = spec.lay
+    offs = oracle.budget_idx_offsets(spec, out["ktok"])
+    cl = [p["h"][7:11].mean(0), p["h"][14:16].mean(0)]
+    nt = p["n_tok"].reshape(-1)
+    kt = p["k"].reshape(-1)
+    for sgi in range(8):
+        e, n, km, r0 = sgi // 4, int(nt[sgi]), int(kt[sgi]), int(lay["row_off"][sgi])
+        if n == 0:
+            continue
+        kk = out["ktok"][r0:r0 + n]
+        assert kk.sum() == km * n                                       # B_m = K_m |I_m|
+        if km in (0, G):
+            assert np.all(kk == km)
+            continue
+        # priorities pi = u . softmax(W_re h + b_re), computed here with scipy
+        a = scipy.special.softmax(p["h"][r0:r0 + n] @ p["W_re"].T + p["b_re"], axis=1)
+        pri = a @ p["u"]
+        assert np.max(np.abs(out["pri"][r0:r0 + n] - pri)) < 1e-12
+        order = np.argsort(-pri, kind="stable")
+        assert list(kk[order]) == list(oracle.budget_shares(n, km * n, G))
+        for i in range(n):
+            r = r0 + i
+            gam = (p["W_v"] @ p["h"][r] + p["b_v"]) + 0.1 * (p["W_role"] @ a[i]) + \
+                0.1 * (p["W_l"] @ cl[e] + p["b_l"])
+            assert np.max(np.abs(out["gamma"][r] - gam)) < 1e-12
+            best = max(itertools.combinations(range(G), int(kk[i])), key=lambda s: sum(gam[list(s)]))
+            sel = out["idx"][offs[r]:offs[r] + int(kk[i])]
+            assert tuple(sel) == tuple(sorted(best))
+
+
+def test_budget_equal_counts_match_fixed_k_packing(oracle):
+    # forcing K_i = K_m for every token must reproduce the fixed-k layout of
+    # the C packer exactly (the numpy packer is written independently)
+    rng = np.random.default_rng(43)
+    G = 4
+    p = _budget_problem(rng, n_tok=((5, 3, 0, 0),), k=((2, 1, G, 0),), G=G)
+    rows = int(np.sum(p["n_tok"]))
+    kf = np.array([2] * 5 + [1] * 3, np.int32)
+    spec, out = _route_budget(oracle, p, k_force=kf)
+    packed = oracle.pack_layer_budget(spec, p["v"], p["R"], out["idx"], out["ktok"])
+    c = oracle.compress_layer(spec, p["h"], p["v"], p["R"], p["W_re"], p["b_re"], np.zeros((1, 2 * spec.d + spec.C)),
+                              np.zeros(1), np.zeros((G, 1)), np.zeros(G), 0.1, 0.1, idx_force=out["idx"])
+    assert rows == 8
+    assert np.max(np.abs(packed - c["packed"])) < 1e-12
+    o1 = oracle.attend_layer_budget(spec, p["q"], p["K"], packed, out["idx"], out["ktok"], p["R"])
+    o2 = oracle.attend_layer(spec, p["q"], p["K"], c["packed"], c["idx"], p["R"])
+    assert np.max(np.abs(o1 - o2)) < 1e-12
+
+
+def test_budget_every_count_vector_equals_dense_over_routed_values(oracle):
+    # every admissible per-token count vector (sum = B_m, 0..S) on a tiny
+    # segment, each with the router's best subsets: attention equals dense
+    # attention over explicitly built R M_j R^T v_j
+    rng = np.random.default_rng(44)
+    G = 4
+    p = _budget_problem(rng, n_tok=((3, 0, 0, 0),), k=((2, G, G, G),), G=G)
+    for kf in itertools.product(range(G + 1), repeat=3):
+        if sum(kf) != 6:
+            continue
+        spec, out = _route_budget(oracle, p, k_force=np.array(kf, np.int32))
+        offs = oracle.budget_idx_offsets(spec, out["ktok"])
+        packed = oracle.pack_layer_budget(spec, p["v"], p["R"], out["idx"], out["ktok"])
+        o = oracle.attend_layer_budget(spec, p["q"], p["K"], packed, out["idx"], out["ktok"], p["R"])
+        masks = {r: tuple(out["idx"][offs[r]:offs[r] + kf[r]]) for r in range(3)}
+        ref = dense_attention(p, _vtil(p, masks))
+        assert np.max(np.abs(o - ref)) <= 1e-12, kf
+
+
+def test_budget_forced_counts_must_meet_the_budget(oracle):
+    rng = np.random.default_rng(45)
+    p = _budget_problem(rng, n_tok=((3, 0, 0, 0),), k=((2, 4, 4, 4),))
+    with pytest.raises(ValueError):
+        _route_budget(oracle, p, k_force=np.array([2, 2, 1], np.int32))   # sums to 5, not 6
+    with pytest.raises(ValueError):
+        _route_budget(oracle, p, k_force=np.array([5, 1, 0], np.int32))   # 5 > S
