@@ -437,6 +437,39 @@ def run_ours(args):
     assert code == 0, f"device status {code}"
     add_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_add)
 
+    # ---- per-token budgets (Sec. 3.5): compress_budget + attend_budget on
+    # the same cache (segment budgets B_m = K_m n), timed on their own -------
+    u_pri = torch.from_numpy(synth.gen_priority(wl_add)).to(dev)
+    k_tok = torch.empty((wl.L, max(wl.rows, 1)), dtype=torch.uint8, device=dev)
+
+    def compress_budget():
+        rs_add.compress_budget(d["h"], d["v"], d["R"], W_re_add, b_re_add, add["W_v"], add["b_v"], add["W_role"],
+                               add["W_l"], add["b_l"], u_pri, wl.alpha_role, wl.alpha_lang, packed=packed,
+                               idx=idx, k_tok=k_tok)
+
+    def attend_budget():
+        rs_add.attend_budget(d["q"], d["K"], packed, idx, k_tok, d["R"], o=o)
+
+    for _ in range(3):
+        compress_budget()
+        attend_budget()
+    torch.cuda.synchronize()
+    ev_bud = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+               torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        if flush_buf is not None:
+            flush_buf.fill_(i & 0xFF)
+        ev_bud[i][0].record(stream)
+        compress_budget()
+        ev_bud[i][1].record(stream)
+        attend_budget()
+        ev_bud[i][2].record(stream)
+    torch.cuda.synchronize()
+    code, _ = rs_add.device_status()
+    assert code == 0, f"device status {code}"
+    bud_c_ms = statistics.mean(a.elapsed_time(b) for a, b, c in ev_bud)
+    bud_a_ms = statistics.mean(b.elapsed_time(c) for a, b, c in ev_bud)
+
     # ---- end to end through the public API from pinned host buffers --------
     act = ("h", "v", "K", "q")
     host = {}
@@ -491,6 +524,10 @@ def run_ours(args):
     cab = compress_additive_bytes(wl, C_ADD)
     comp_add = {"ms": add_ms, "role_dim": C_ADD, "algorithmic_bytes": cab, "GB/s": cab / (add_ms / 1e3) / 1e9,
                 "frac": cab / (add_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
+    budget = {"role_dim": C_ADD, "compress_ms": bud_c_ms, "compress_GB/s": cab / (bud_c_ms / 1e3) / 1e9,
+              "attend_ms": bud_a_ms, "attend_GB/s": ab / (bud_a_ms / 1e3) / 1e9,
+              "attend_frac": ab / (bud_a_ms / 1e3) / 1e9 / peaks["hbm_gbs"],
+              "query_tokens_per_s_per_layer": qtok / ((bud_c_ms + bud_a_ms) / 1e3)}
 
     clocks = clk.summary()
     line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
@@ -501,7 +538,7 @@ def run_ours(args):
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                     "ms_per_step": e2e_ms},
             "gpu_launches": launches,
-            "roofline": roof, "compress": comp, "compress_additive": comp_add,
+            "roofline": roof, "compress": comp, "compress_additive": comp_add, "budget": budget,
             "clocks": {"sm_mhz": clocks["sm_mhz"], "sm_max_mhz": clocks["sm_max_mhz"],
                        "reasons": clocks["reasons"], "samples": clocks["samples"]}}
     if ws == 1 and rank == 0 and not args.no_cpu_baseline:

@@ -240,6 +240,67 @@ rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
                               const void *R, float softmax_scale, void *o, void *workspace,
                               size_t ws_bytes, void *stream);
 
+/*
+ * Per-token value budgets (Sec. 3.5) with the additive routing score
+ * (Sec. 3.4, as in rolesub_compress_additive).
+ *
+ * In a segment of n tokens whose plan entry has k = K_m with 0 < K_m < S,
+ * the tokens share B_m = K_m n groups: token i keeps K_i groups,
+ * 0 <= K_i <= S, sum_i K_i = B_m, more for higher role-derived priority.
+ * The paper states those constraints but no formula; this library's
+ * allocator:
+ *   pi_i = u . a_i, a_i = softmax(W_re h_i + b_re)   (Eq. latentrole)
+ *   rank the tokens by pi (higher first; ties: lower token index); rank r
+ *   has weight n - r; real shares x_r = min(S, lambda (n - r)) with
+ *   sum x = B_m; K = x rounded by largest remainders (ties: better rank).
+ * Priorities and scores are fp32 on the device; tokens whose priorities lie
+ * within rounding of each other may exchange ranks.
+ * Token i keeps its K_i largest scores (ties: lower group index), indices
+ * ascending. Segments with K_m = S keep everything, K_m = 0 nothing.
+ *
+ * Cache layout: the plan's segment regions are unchanged (B_m groups per
+ * head, B_m index bytes); inside a segment token i's indices start at
+ * idx_off + sum_{j<i} K_j and head h's values at
+ * packed_off + (h B_m + sum_{j<i} K_j) d_s.
+ *
+ * Inputs: as rolesub_compress_additive, plus
+ *   u      [L][C] float32   priority vector of each layer's allocator
+ * Outputs: packed_v, idx as above and
+ *   k_tok  [L][rows_per_layer] uint8   K_i of every cache row (the attention
+ *          call needs it)
+ * workspace: at least rolesub_budget_workspace_size bytes (the common
+ * workspace followed by the router's scores and priorities).
+ * Supported geometry: bf16, d_h = 128, S = 16, S + C <= 256, d % 64 == 0,
+ * segments of at most 8192 tokens; otherwise ROLESUB_EUNSUPPORTED.
+ * Other errors: as rolesub_compress.
+ */
+rolesub_status rolesub_budget_workspace_size(const rolesub_shape *shape, const void *plan_host,
+                                             size_t *bytes);
+rolesub_status rolesub_compress_budget(const rolesub_shape *shape, const void *plan_host,
+                                       const void *plan_dev, const void *h, const void *v,
+                                       const void *R, const void *W_re, const float *b_re,
+                                       const void *W_v, const float *b_v, const void *W_role,
+                                       const void *W_l, const float *b_l, const float *u,
+                                       float alpha_role, float alpha_lang, void *packed_v,
+                                       uint8_t *idx, uint8_t *k_tok, void *workspace,
+                                       size_t ws_bytes, void *stream);
+
+/*
+ * rolesub_attend over a cache written by rolesub_compress_budget: the same
+ * arguments plus its k_tok. Counts above S, counts that overrun a segment's
+ * B_m and stored indices >= S are reported through the device status word
+ * (ROLESUB_EDEVICE) and that row contributes no values. workspace:
+ * rolesub_workspace_size bytes. Geometry: as rolesub_compress_budget.
+ */
+rolesub_status rolesub_attend_budget(const rolesub_shape *shape, const void *plan_host,
+                                     const void *plan_dev, const void *q, int64_t q_layer_stride,
+                                     int64_t q_row_stride, int64_t q_head_stride, const void *K,
+                                     int64_t k_layer_stride, int64_t k_row_stride,
+                                     int64_t k_head_stride, const void *packed_v,
+                                     const uint8_t *idx, const uint8_t *k_tok, const void *R,
+                                     float softmax_scale, void *o, void *workspace,
+                                     size_t ws_bytes, void *stream);
+
 /* Waits for the stream, then reads the workspace's status word:
  * *code_out = 0 when no kernel reported bad data, else a ROLESUB_E* code.
  * *detail_out (may be NULL) receives the first reported item. */

@@ -39,6 +39,11 @@ bool shape_ok(const rolesub_shape *s)
     return true;
 }
 
+// The per-token budget path (Sec. 3.5): bf16, d_h = 128, S = 16 (the
+// tensor-core rotation, attention and additive router), S + C <= 256,
+// d % 64 == 0, and segments of at most 8192 tokens.
+bool budget_supported(const rolesub_shape *s, const PlanView &pv);
+
 struct Sizes {
     size_t header, segs, eps, row_seg, routed, stored, tiles, total;
 };
@@ -128,6 +133,14 @@ Workspace carve(const WsSizes &w, void *base)
 }
 
 rolesub_status from_cuda(cudaError_t e) { return e == cudaSuccess ? ROLESUB_OK : ROLESUB_ECUDA; }
+
+bool budget_supported(const rolesub_shape *s, const PlanView &pv)
+{
+    if (!rs::rotate_tc_supported(s) || !rs::attend_tc_supported(s) || !rs::additive_tc_supported(s)) return false;
+    for (int i = 0; i < pv.hdr->num_segments; ++i)
+        if (pv.segs[i].n_tokens > 8192) return false;
+    return true;
+}
 
 }  // namespace
 
@@ -365,12 +378,25 @@ rolesub_status rolesub_compress_additive(const rolesub_shape *shape, const void 
     return from_cuda(rs::launch_rotate_pack(a));
 }
 
-rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
-                              const void *plan_dev, const void *q, int64_t q_ls, int64_t q_rs,
-                              int64_t q_hs, const void *K, int64_t k_ls, int64_t k_rs,
-                              int64_t k_hs, const void *packed_v, const uint8_t *idx,
-                              const void *R, float softmax_scale, void *o, void *workspace,
-                              size_t ws_bytes, void *stream)
+}  // extern "C"
+
+namespace {
+
+// Scores and priorities of the budget path's router: [L][rows][20] fp32
+// after the common workspace.
+size_t budget_scores_bytes(const rolesub_shape *shape, const rolesub_plan *p)
+{
+    return align_up(sizeof(float) * rs::kScoreStride * (size_t)shape->num_layers * (size_t)p->rows_per_layer,
+                    kAlign);
+}
+
+// Shared by rolesub_attend (k_tok = NULL: the plan's k per segment) and
+// rolesub_attend_budget (per-token counts).
+rolesub_status attend_common(const rolesub_shape *shape, const void *plan_host, const void *plan_dev,
+                             const void *q, int64_t q_ls, int64_t q_rs, int64_t q_hs, const void *K, int64_t k_ls,
+                             int64_t k_rs, int64_t k_hs, const void *packed_v, const uint8_t *idx,
+                             const uint8_t *k_tok, bool budget, const void *R, float softmax_scale, void *o,
+                             void *workspace, size_t ws_bytes, void *stream)
 {
     if (!shape_ok(shape)) return ROLESUB_EINVAL;
     PlanView pv;
@@ -383,6 +409,7 @@ rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
         if (!p || !aligned16(p)) return ROLESUB_EINVAL;
     if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
     if (P.idx_bytes_per_layer > 0 && !idx) return ROLESUB_EINVAL;
+    if (budget && P.rows_per_layer > 0 && !k_tok) return ROLESUB_EINVAL;
     const int64_t sm = 16 / elem_bytes(shape->dtype);
     const int64_t strides[] = {q_ls, q_rs, q_hs, k_ls, k_rs, k_hs};
     for (int64_t x : strides)
@@ -391,6 +418,7 @@ rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
     const WsSizes w = ws_sizes(shape, pv.hdr);
     if (ws_bytes < w.total) return ROLESUB_EINVAL;
     if (!rs::attend_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    if (budget && !budget_supported(shape, pv)) return ROLESUB_EUNSUPPORTED;
     rs::AttendArgs a;
     a.shape = shape;
     a.plan = pv;
@@ -409,7 +437,99 @@ rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
     a.scale = softmax_scale;
     a.o = o;
     a.stream = (cudaStream_t)stream;
+    if (budget) {
+        a.k_tok = k_tok;
+        return from_cuda(rs::launch_attend_tc(a));
+    }
     return from_cuda(rs::launch_attend(a));
+}
+
+}  // namespace
+
+extern "C" {
+
+rolesub_status rolesub_attend(const rolesub_shape *shape, const void *plan_host,
+                              const void *plan_dev, const void *q, int64_t q_ls, int64_t q_rs,
+                              int64_t q_hs, const void *K, int64_t k_ls, int64_t k_rs,
+                              int64_t k_hs, const void *packed_v, const uint8_t *idx,
+                              const void *R, float softmax_scale, void *o, void *workspace,
+                              size_t ws_bytes, void *stream)
+{
+    return attend_common(shape, plan_host, plan_dev, q, q_ls, q_rs, q_hs, K, k_ls, k_rs, k_hs, packed_v, idx,
+                         nullptr, false, R, softmax_scale, o, workspace, ws_bytes, stream);
+}
+
+rolesub_status rolesub_attend_budget(const rolesub_shape *shape, const void *plan_host,
+                                     const void *plan_dev, const void *q, int64_t q_ls, int64_t q_rs,
+                                     int64_t q_hs, const void *K, int64_t k_ls, int64_t k_rs,
+                                     int64_t k_hs, const void *packed_v, const uint8_t *idx,
+                                     const uint8_t *k_tok, const void *R, float softmax_scale, void *o,
+                                     void *workspace, size_t ws_bytes, void *stream)
+{
+    return attend_common(shape, plan_host, plan_dev, q, q_ls, q_rs, q_hs, K, k_ls, k_rs, k_hs, packed_v, idx,
+                         k_tok, true, R, softmax_scale, o, workspace, ws_bytes, stream);
+}
+
+rolesub_status rolesub_budget_workspace_size(const rolesub_shape *shape, const void *plan_host, size_t *bytes)
+{
+    if (!shape_ok(shape) || !bytes) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, nullptr, &pv);
+    if (st != ROLESUB_OK) return st;
+    *bytes = ws_sizes(shape, pv.hdr).total + budget_scores_bytes(shape, pv.hdr);
+    return ROLESUB_OK;
+}
+
+rolesub_status rolesub_compress_budget(const rolesub_shape *shape, const void *plan_host,
+                                       const void *plan_dev, const void *h, const void *v,
+                                       const void *R, const void *W_re, const float *b_re,
+                                       const void *W_v, const float *b_v, const void *W_role,
+                                       const void *W_l, const float *b_l, const float *u,
+                                       float alpha_role, float alpha_lang, void *packed_v,
+                                       uint8_t *idx, uint8_t *k_tok, void *workspace,
+                                       size_t ws_bytes, void *stream)
+{
+    if (!shape_ok(shape)) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, plan_dev, &pv);
+    if (st != ROLESUB_OK) return st;
+    if (!plan_dev) return ROLESUB_EINVAL;
+    const void *ptrs[] = {h, v, R, W_re, b_re, W_v, b_v, W_role, W_l, b_l, u, workspace};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    const rolesub_plan &P = *pv.hdr;
+    if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
+    if (P.idx_bytes_per_layer > 0 && (!idx || !aligned16(idx))) return ROLESUB_EINVAL;
+    if (P.rows_per_layer > 0 && !k_tok) return ROLESUB_EINVAL;
+    if (!isfinite(alpha_role) || !isfinite(alpha_lang)) return ROLESUB_EINVAL;
+    if (!budget_supported(shape, pv)) return ROLESUB_EUNSUPPORTED;
+    const WsSizes w = ws_sizes(shape, pv.hdr);
+    const size_t sb = budget_scores_bytes(shape, pv.hdr);
+    if (ws_bytes < w.total + sb) return ROLESUB_EINVAL;
+    rs::CompressArgs a{};
+    a.shape = shape;
+    a.plan = pv;
+    a.ws = carve(w, workspace);
+    a.h = h;
+    a.v = v;
+    a.R = R;
+    a.W_re = W_re;
+    a.b_re = b_re;
+    a.alpha_role = alpha_role;
+    a.alpha_lang = alpha_lang;
+    a.packed = packed_v;
+    a.idx = idx;
+    a.stream = (cudaStream_t)stream;
+    float *scores = reinterpret_cast<float *>(static_cast<char *>(workspace) + w.total);
+    rs::AdditiveWeights wt{W_v, W_role, W_l, b_v, b_l};
+    wt.u = u;
+    wt.scores = scores;
+    cudaError_t e = rs::launch_router_additive(a, wt);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    e = rs::launch_budget_select(a, scores, k_tok);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    a.records_ready = true;
+    return from_cuda(rs::launch_rotate_pack(a));
 }
 
 rolesub_status rolesub_get_device_status(const void *workspace, void *stream, int32_t *code_out,

@@ -717,8 +717,10 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
         sms = 152;
     // per-row records (kept groups, packed offset) from the caller's indices
     uint4 *recs = reinterpret_cast<uint4 *>(a.ws.row_store);
-    err = launch_row_store(a.plan, L, const_cast<uint8_t *>(a.idx), P.idx_bytes_per_layer, false, recs, a.ws.status,
-                           a.stream);
+    err = a.k_tok ? launch_row_store_budget(a.plan, L, a.idx, P.idx_bytes_per_layer, a.k_tok, recs, a.ws.status,
+                                            a.stream)
+                  : launch_row_store(a.plan, L, const_cast<uint8_t *>(a.idx), P.idx_bytes_per_layer, false, recs,
+                                     a.ws.status, a.stream);
     if (err != cudaSuccess) return err;
     const int qtiles = (P.max_query_tokens + kQRows - 1) / kQRows;
     const float scale = a.scale > 0.f ? a.scale : 1.0f / sqrtf((float)kDh);

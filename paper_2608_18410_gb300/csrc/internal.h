@@ -43,6 +43,7 @@ struct CompressArgs {
     void *packed;
     uint8_t *idx;
     cudaStream_t stream;
+    bool records_ready = false;   // ws.row_store already holds the store records
 };
 
 // Weights of the additive routing score (Sec. 3.4, Eq. routingscore):
@@ -51,7 +52,13 @@ struct CompressArgs {
 struct AdditiveWeights {
     const void *W_v, *W_role, *W_l;
     const float *b_v, *b_l;
+    // score mode (per-token budgets, Sec. 3.5): u [L][C] float32 gives the
+    // priority pi = u . a; gamma and pi of every routed row go to scores
+    // [L][rows][kScoreStride] (gamma at 0..S-1, pi at S) instead of a top-k
+    const float *u = nullptr;
+    float *scores = nullptr;
 };
+constexpr int kScoreStride = 20;   // floats per row: 16 scores, pi, padding to 16 bytes
 
 struct AttendArgs {
     const rolesub_shape *shape;
@@ -63,6 +70,7 @@ struct AttendArgs {
     float scale;
     void *o;
     cudaStream_t stream;
+    const uint8_t *k_tok = nullptr;   // per-token kept counts (budget cache), or fixed k
 };
 
 // Router: language pool + per-episode bias, router GEMM, epilogue/top-k.
@@ -72,6 +80,7 @@ cudaError_t launch_lang_pool(const CompressArgs &a);
 // Additive router: language term per episode, then scores and top-k per
 // routed row (tcgen05 for bf16, S = 16, S + C <= 256, d % 64 == 0).
 bool router_additive_supported(const rolesub_shape *s);
+bool additive_tc_supported(const rolesub_shape *s);
 cudaError_t launch_router_additive(const CompressArgs &a, const AdditiveWeights &w);
 // Rotation z = R_h^T v and packing of the kept groups.
 cudaError_t launch_rotate_pack(const CompressArgs &a);
@@ -91,6 +100,14 @@ cudaError_t launch_attend(const AttendArgs &a);
 // Routed attention on tcgen05/TMA (bf16, d_h = 128, S = 16).
 bool attend_tc_supported(const rolesub_shape *s);
 cudaError_t launch_attend_tc(const AttendArgs &a);
+
+// Per-token budgets (Sec. 3.5): from the scores and priorities of score
+// mode, the counts K_i of every routed segment, the kept groups at prefix
+// offsets, k_tok and the store records (also for k = 0 and k = S segments).
+cudaError_t launch_budget_select(const CompressArgs &a, const float *scores, uint8_t *k_tok);
+// Store records of a budget cache from its indices and per-token counts.
+cudaError_t launch_row_store_budget(const PlanView &pv, int L, const uint8_t *idx, int64_t idx_per_layer,
+                                    const uint8_t *k_tok, uint4 *recs, int32_t *status, cudaStream_t stream);
 
 // Adds n to the process-wide launch counter (rolesub_launch_count).
 void count_launches(int n);

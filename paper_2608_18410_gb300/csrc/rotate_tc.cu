@@ -261,8 +261,10 @@ cudaError_t launch_rotate_tc(const CompressArgs &a)
     const int per = (ntiles + splits - 1) / splits;
     splits = (ntiles + per - 1) / per;
     uint4 *meta = reinterpret_cast<uint4 *>(a.ws.row_store);
-    err = launch_row_store(a.plan, L, a.idx, P.idx_bytes_per_layer, true, meta, a.ws.status, a.stream);
-    if (err != cudaSuccess) return err;
+    if (!a.records_ready) {
+        err = launch_row_store(a.plan, L, a.idx, P.idx_bytes_per_layer, true, meta, a.ws.status, a.stream);
+        if (err != cudaSuccess) return err;
+    }
     k_rotate_tc<<<dim3(H, L, splits), kThreads, kSmemBytes, a.stream>>>(
         tv, tr, meta, rows, H, per, ntiles, (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
     count_launches(1);

@@ -462,8 +462,8 @@ k_router_epilogue(const float *__restrict__ logits, PlanDev plan, int64_t M, int
     const int k = sg.k;
     const bool keep = lane < G && rank < k;
     const unsigned ball = __ballot_sync(0xffffffffu, keep);
-    if (keep) {
-        const int pos = __popc(ball & ((1u << lane) - 1u));
+    const int pos = __popc(ball & ((1u << lane) - 1u));
+    if (keep && pos < k) {   // pos < k: NaN scores rank 0 and must not overflow the row
         const int64_t ti = row - sg.token_row;
         idx[(size_t)l * idx_per_layer + sg.idx_off + ti * k + pos] = (uint8_t)lane;
     }

@@ -163,8 +163,8 @@ k_router_add_simt(const T *__restrict__ h, PlanDev plan, int64_t M, int64_t rows
     const int k = sg.k;
     const bool keep = lane < G && rank < k;
     const unsigned ball = __ballot_sync(0xffffffffu, keep);
-    if (keep) {
-        const int pos = __popc(ball & ((1u << lane) - 1u));
+    const int pos = __popc(ball & ((1u << lane) - 1u));
+    if (keep && pos < k) {   // pos < k: NaN scores rank 0 and must not overflow the row
         idx[(size_t)l * idx_per_layer + sg.idx_off + (int64_t)(r - sg.token_row) * k + pos] = (uint8_t)lane;
     }
 }
@@ -189,7 +189,8 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
                 const __grid_constant__ CUtensorMap tm_wre, PlanDev plan, int64_t rows, int d, int C, int E,
                 int nb, int stages, const float *__restrict__ b_v, const float *__restrict__ b_re,
                 const bf16 *__restrict__ W_role, const float *__restrict__ beta, float alpha_role,
-                uint8_t *__restrict__ idx, int64_t idx_per_layer, int32_t *status)
+                uint8_t *__restrict__ idx, int64_t idx_per_layer, const float *__restrict__ u_pri,
+                float *__restrict__ scores, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ uint32_t tmem_slot;
@@ -203,7 +204,7 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
     const int nkb = d / 64;
     const uint32_t stage_bytes = kTileA + (uint32_t)nb * 128u;
     const uint32_t off_role = (uint32_t)stages * stage_bytes;
-    const uint32_t off_bar = (off_role + 4u * kTG * (uint32_t)C + 7u) & ~7u;
+    const uint32_t off_bar = (off_role + 4u * (kTG + 1) * (uint32_t)C + 7u) & ~7u;
     const uint32_t bar_full = sb + off_bar, bar_empty = bar_full + 8u * kTMaxStages,
                    bar_acc = bar_empty + 8u * kTMaxStages;
     const uint32_t ncols = tmem_cols_for(nb);
@@ -225,6 +226,8 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
             reinterpret_cast<uint32_t *>(sp + s * stage_bytes + kTileA + (kTG + C) * 128)[i] = 0u;
     float *wr = reinterpret_cast<float *>(sp + off_role);
     for (int i = tid; i < kTG * C; i += kTThreads) wr[i] = __bfloat162float(W_role[(size_t)l * kTG * C + i]);
+    float *wu = wr + kTG * C;   // priority vector u (score mode), else zeros
+    for (int i = tid; i < C; i += kTThreads) wu[i] = scores ? u_pri[(size_t)l * C + i] : 0.f;
     fence_async_smem();
     __syncthreads();
     if (warp == 0) {
@@ -286,11 +289,12 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
         // columns [0, S): token scores; [S, S + C): role logits. The role
         // softmax runs online over 32-column chunks: a running max mx, the
         // running sum z of exp(logit - mx) and acc_s = sum_c W_role[s][c]
-        // exp(logit_c - mx), both rescaled when mx grows.
+        // exp(logit_c - mx), all rescaled when mx grows (accp: the same sum
+        // with the priority vector u, pi = u . a, Sec. 3.5).
         float gam[kTG], acc[kTG];
 #pragma unroll
         for (int s = 0; s < kTG; ++s) acc[s] = 0.f;
-        float mx = -INFINITY, z = 0.f;
+        float mx = -INFINITY, z = 0.f, accp = 0.f;
 #pragma unroll 1
         for (int c0 = 0; c0 < kTG + C; c0 += 32) {
             uint32_t sr[32];
@@ -313,6 +317,7 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
             const float nm = fmaxf(mx, cm);
             const float rescale = expf(mx - nm);
             z *= rescale;
+            accp *= rescale;
 #pragma unroll
             for (int s = 0; s < kTG; ++s) acc[s] *= rescale;
 #pragma unroll
@@ -321,6 +326,7 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
                 if (c >= 0 && c < C) {
                     const float e = expf(lg[j] - nm);
                     z += e;
+                    accp = fmaf(wu[c], e, accp);
 #pragma unroll
                     for (int s = 0; s < kTG; ++s) acc[s] = fmaf(wr[s * C + c], e, acc[s]);
                 }
@@ -332,16 +338,27 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
             const float inv = 1.f / z;
 #pragma unroll
             for (int s = 0; s < kTG; ++s) gam[s] += alpha_role * (acc[s] * inv) + __ldg(be + s);
-            const int k = sg.k;
-            uint8_t *dst = idx + (int64_t)l * idx_per_layer + sg.idx_off + (r - sg.token_row) * k;
-            int pos = 0;
+            if (scores) {
+                // score mode (per-token budgets): gamma and pi to the
+                // workspace, the selection runs once the segment's counts
+                // are known
+                float4 *dst = reinterpret_cast<float4 *>(scores + ((int64_t)l * rows + r) * kScoreStride);
 #pragma unroll
-            for (int g = 0; g < kTG; ++g) {
-                int rank = 0;
+                for (int q = 0; q < kTG / 4; ++q)
+                    dst[q] = make_float4(gam[4 * q], gam[4 * q + 1], gam[4 * q + 2], gam[4 * q + 3]);
+                dst[kTG / 4] = make_float4(accp * inv, 0.f, 0.f, 0.f);
+            } else {
+                const int k = sg.k;
+                uint8_t *dst = idx + (int64_t)l * idx_per_layer + sg.idx_off + (r - sg.token_row) * k;
+                int pos = 0;
 #pragma unroll
-                for (int g2 = 0; g2 < kTG; ++g2)
-                    rank += (gam[g2] > gam[g] || (gam[g2] == gam[g] && g2 < g)) ? 1 : 0;
-                if (rank < k) dst[pos++] = (uint8_t)g;
+                for (int g = 0; g < kTG; ++g) {
+                    int rank = 0;
+#pragma unroll
+                    for (int g2 = 0; g2 < kTG; ++g2)
+                        rank += (gam[g2] > gam[g] || (gam[g2] == gam[g] && g2 < g)) ? 1 : 0;
+                    if (rank < k && pos < k) dst[pos++] = (uint8_t)g;   // pos < k: NaN-safe
+                }
             }
         }
     }
@@ -353,11 +370,15 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
     }
 }
 
+}  // namespace
+
 bool additive_tc_supported(const rolesub_shape *s)
 {
     const int d = s->num_heads * s->head_dim;
     return s->dtype == ROLESUB_BF16 && s->num_groups == kTG && s->role_dim <= 256 - kTG && d % 64 == 0;
 }
+
+namespace {
 
 template <class T>
 cudaError_t launch_additive_t(const CompressArgs &a, const AdditiveWeights &w)
@@ -385,8 +406,8 @@ cudaError_t launch_additive_t(const CompressArgs &a, const AdditiveWeights &w)
         const int nb = (G + C + 15) / 16 * 16;
         const uint32_t stage_bytes = kTileA + 128u * (uint32_t)nb;
         const int stages = std::min<int>(kTMaxStages, (int)(kRingBudget / stage_bytes));
-        const uint32_t smem =
-            (uint32_t)stages * stage_bytes + 4u * kTG * (uint32_t)C + 8u + 8u * (2 * kTMaxStages + 1) + 1024u;
+        const uint32_t smem = (uint32_t)stages * stage_bytes + 4u * (kTG + 1) * (uint32_t)C + 8u +
+                              8u * (2 * kTMaxStages + 1) + 1024u;
         const int64_t rows = P.rows_per_layer;
         CUtensorMap th, twv, twre;
         {
@@ -411,10 +432,11 @@ cudaError_t launch_additive_t(const CompressArgs &a, const AdditiveWeights &w)
         if (err != cudaSuccess) return err;
         k_router_add_tc<<<dim3((unsigned)P.num_route_tiles, L), kTThreads, smem, a.stream>>>(
             th, twv, twre, pd, rows, d, C, E, nb, stages, w.b_v, a.b_re, (const bf16 *)w.W_role, a.ws.lang_bias,
-            a.alpha_role, a.idx, P.idx_bytes_per_layer, a.ws.status);
+            a.alpha_role, a.idx, P.idx_bytes_per_layer, w.u, w.scores, a.ws.status);
         count_launches(1);
         return cudaGetLastError();
     }
+    if (w.scores) return cudaErrorInvalidValue;   // score mode: tensor-core path only
     const size_t smem = (size_t)8 * (G + C) * sizeof(float);
     if (smem > 48 * 1024) {
         err = cudaFuncSetAttribute(k_router_add_simt<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -278,7 +278,7 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
 #pragma unroll
                 for (int g2 = 0; g2 < kG; ++g2)
                     rank += (gam[g2] > gam[g] || (gam[g2] == gam[g] && g2 < g)) ? 1 : 0;
-                if (rank < k) dst[pos++] = (uint8_t)g;
+                if (rank < k && pos < k) dst[pos++] = (uint8_t)g;   // pos < k: NaN-safe
             }
         }
     }

@@ -30,7 +30,8 @@ STATUS = {0: "ROLESUB_OK", 1: "ROLESUB_EINVAL", 2: "ROLESUB_EUNSUPPORTED", 3: "R
 EXPORTS = ("rolesub_plan_size", "rolesub_layout_plan", "rolesub_workspace_size",
            "rolesub_compress", "rolesub_attend", "rolesub_get_device_status",
            "rolesub_reset_device_status", "rolesub_status_string", "rolesub_version",
-           "rolesub_launch_count", "rolesub_compress_static", "rolesub_compress_additive")
+           "rolesub_launch_count", "rolesub_compress_static", "rolesub_compress_additive",
+           "rolesub_budget_workspace_size", "rolesub_compress_budget", "rolesub_attend_budget")
 
 STATIC_SCRATCH_BYTES = 8 << 20
 
@@ -110,6 +111,12 @@ def lib():
                                               + [_vp, _vp, _vp])
         L.rolesub_compress_additive.argtypes = ([sp, _vp, _vp] + [_vp] * 10 + [ctypes.c_float, ctypes.c_float]
                                                 + [_vp, _vp, _vp, ctypes.c_size_t, _vp])
+        L.rolesub_budget_workspace_size.argtypes = [sp, _vp, _szp]
+        L.rolesub_compress_budget.argtypes = ([sp, _vp, _vp] + [_vp] * 11 + [ctypes.c_float, ctypes.c_float]
+                                              + [_vp, _vp, _vp, _vp, ctypes.c_size_t, _vp])
+        L.rolesub_attend_budget.argtypes = ([sp, _vp, _vp, _vp] + [ctypes.c_int64] * 3 + [_vp]
+                                            + [ctypes.c_int64] * 3 + [_vp, _vp, _vp, _vp, ctypes.c_float, _vp,
+                                                                      _vp, ctypes.c_size_t, _vp])
         L.rolesub_launch_count.argtypes = []
         L.rolesub_launch_count.restype = ctypes.c_uint64
         for name in EXPORTS:
@@ -186,6 +193,12 @@ class Plan:
         self.dev = torch.from_numpy(self.host[: self.hdr.total_bytes].copy()).to(device)
         return self.dev
 
+    def budget_workspace_size(self):
+        sz = ctypes.c_size_t(0)
+        _check("rolesub_budget_workspace_size", lib().rolesub_budget_workspace_size(
+            ctypes.byref(self.shape), self.host_ptr, ctypes.byref(sz)))
+        return int(sz.value)
+
     def workspace_size(self):
         sz = ctypes.c_size_t(0)
         _check("rolesub_workspace_size", lib().rolesub_workspace_size(
@@ -213,6 +226,25 @@ def rolesub_compress_additive(shape, plan: Plan, plan_dev, h, v, R, W_re, b_re, 
         ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(h), _ptr(v), _ptr(R), _ptr(W_re),
         _ptr(b_re), _ptr(W_v), _ptr(b_v), _ptr(W_role), _ptr(W_l), _ptr(b_l), float(alpha_role),
         float(alpha_lang), _ptr(packed_v), _ptr(idx), _ptr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def rolesub_compress_budget(shape, plan: Plan, plan_dev, h, v, R, W_re, b_re, W_v, b_v, W_role, W_l, b_l, u,
+                            alpha_role, alpha_lang, packed_v, idx, k_tok, workspace, ws_bytes=None, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size() if ws_bytes is None else ws_bytes
+    _check("rolesub_compress_budget", lib().rolesub_compress_budget(
+        ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(h), _ptr(v), _ptr(R), _ptr(W_re),
+        _ptr(b_re), _ptr(W_v), _ptr(b_v), _ptr(W_role), _ptr(W_l), _ptr(b_l), _ptr(u), float(alpha_role),
+        float(alpha_lang), _ptr(packed_v), _ptr(idx), _ptr(k_tok), _ptr(workspace), int(ws_bytes),
+        _stream(stream)))
+
+
+def rolesub_attend_budget(shape, plan: Plan, plan_dev, q, q_strides, K, k_strides, packed_v, idx, k_tok, R,
+                          softmax_scale, o, workspace, ws_bytes=None, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size() if ws_bytes is None else ws_bytes
+    _check("rolesub_attend_budget", lib().rolesub_attend_budget(
+        ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(q), *[int(s) for s in q_strides],
+        _ptr(K), *[int(s) for s in k_strides], _ptr(packed_v), _ptr(idx), _ptr(k_tok), _ptr(R),
+        float(softmax_scale), _ptr(o), _ptr(workspace), int(ws_bytes), _stream(stream)))
 
 
 def rolesub_attend(shape, plan: Plan, plan_dev, q, q_strides, K, k_strides, packed_v, idx, R,
@@ -277,6 +309,9 @@ class RoleSub:
         self.plan = Plan(self.shape, n_tok, k, n_query)
         self.plan_dev = self.plan.to_device(device)
         self.ws_bytes = self.plan.workspace_size()
+        if dtype in ("bf16", BF16) and dh == 128 and G == 16:
+            # room for the per-token budget path's router scores as well
+            self.ws_bytes = max(self.ws_bytes, self.plan.budget_workspace_size())
         self.workspace = torch.zeros(self.ws_bytes, dtype=torch.uint8, device=device)
         self.device = device
         self.tdtype = torch.bfloat16 if dtype in ("bf16", BF16) else torch.float32
@@ -305,6 +340,31 @@ class RoleSub:
                                   W_l, b_l, alpha_role, alpha_lang, packed, idx, self.workspace, self.ws_bytes,
                                   stream)
         return packed, idx
+
+    def compress_budget(self, h, v, R, W_re, b_re, W_v, b_v, W_role, W_l, b_l, u, alpha_role=0.1,
+                        alpha_lang=0.1, packed=None, idx=None, k_tok=None, stream=None):
+        if packed is None or idx is None:
+            packed, idx = self.new_outputs()
+        if k_tok is None:
+            k_tok = self.torch.empty((self.shape.num_layers, max(self.plan.hdr.rows_per_layer, 1)),
+                                     dtype=self.torch.uint8, device=self.device)
+        rolesub_compress_budget(self.shape, self.plan, self.plan_dev, h, v, R, W_re, b_re, W_v, b_v, W_role, W_l,
+                                b_l, u, alpha_role, alpha_lang, packed, idx, k_tok, self.workspace, self.ws_bytes,
+                                stream)
+        return packed, idx, k_tok
+
+    def attend_budget(self, q, K, packed, idx, k_tok, R, softmax_scale=0.0, o=None, stream=None):
+        t = self.torch
+        s = self.shape
+        d = s.num_heads * s.head_dim
+        hdr = self.plan.hdr
+        q_strides = (hdr.q_rows_per_layer * d, d, s.head_dim)
+        k_strides = (hdr.rows_per_layer * d, d, s.head_dim)
+        if o is None:
+            o = t.empty((s.num_layers, max(hdr.q_rows_per_layer, 1), d), dtype=self.tdtype, device=self.device)
+        rolesub_attend_budget(s, self.plan, self.plan_dev, q, q_strides, K, k_strides, packed, idx, k_tok, R,
+                              softmax_scale, o, self.workspace, self.ws_bytes, stream)
+        return o
 
     def attend(self, q, K, packed, idx, R, softmax_scale=0.0, o=None, q_strides=None, k_strides=None,
                stream=None):

@@ -14,6 +14,7 @@ Recipe (one numpy PCG64 stream per tensor block):
   biases  b_re, b1, b2     ~ N(0, 0.02)   float32 (biases are always fp32)
   additive router (gen_additive_weights):
     W_v, W_l ~ N(0, 0.02), W_role ~ N(0, 1), b_v, b_l ~ N(0, 0.02) (fp32)
+  per-token budgets (gen_priority): u ~ N(0, 1) (fp32), one C-vector per layer
   R_h: Haar-random orthogonal d_h x d_h, from the QR factorisation of an
        fp64 N(0, 1) matrix with column signs fixed by sign(diag(R_qr)).
 bf16 tensors are rounded float32 -> bf16 with round-to-nearest-even and are
@@ -33,7 +34,8 @@ KINDS = ("vis", "lang", "prop", "act")
 
 TID = {"h": 1, "v": 2, "q": 3, "K": 4, "R": 5, "W_re": 6, "b_re": 7,
        "W1": 8, "b1": 9, "W2": 10, "b2": 11, "episodes": 12, "near_tie": 13,
-       "packed": 14, "idx": 15, "W_v": 16, "b_v": 17, "W_role": 18, "W_l": 19, "b_l": 20}
+       "packed": 14, "idx": 15, "W_v": 16, "b_v": 17, "W_role": 18, "W_l": 19, "b_l": 20,
+       "u": 21}
 
 
 @dataclasses.dataclass(frozen=True)
@@ -331,6 +333,11 @@ def gen_additive_weights(wl: Workload):
         out["W_l"][layer] = _store(Wl, wl.dtype)
         out["b_l"][layer] = bl
     return out
+
+
+def gen_priority(wl: Workload):
+    """Priority vectors u [L][C] float32 of the per-token budget allocator."""
+    return np.stack([_normal(wl.seed, layer, 0, TID["u"], (wl.C,)) for layer in range(wl.L)]).astype(np.float32)
 
 
 def gen_packed(wl: Workload, packed_elems_per_layer: int, idx_bytes_per_layer: int, seg_table):

@@ -195,3 +195,36 @@ def test_additive_compress_rejects_bad_arguments_before_any_launch(rsm):
     a = list(args)
     a[0], a[1] = ctypes.byref(big), pb.host_ptr
     assert L.rolesub_compress_additive(*a) == 2
+
+
+def test_budget_calls_reject_bad_arguments_before_any_launch(rsm):
+    shape = rsm.make_shape(1, 2, 128, 16, 6, 8, "bf16")
+    plan = rsm.Plan(shape, [[3, 2, 0, 0]], [[4, 16, 16, 16]], [1])
+    L = rsm.lib()
+    fake = 1 << 20    # never dereferenced: validation fails first
+    big = plan.budget_workspace_size()
+    assert big > plan.workspace_size()
+    # shape, plan, plan_dev, h v R W_re b_re W_v b_v W_role W_l b_l u, alphas, packed idx k_tok ws, ws_bytes, stream
+    args = [ctypes.byref(shape), plan.host_ptr, fake] + [fake] * 11 + [0.1, 0.1, fake, fake, fake, fake, big, None]
+    for pos in range(3, 14):
+        a = list(args)
+        a[pos] = None
+        assert L.rolesub_compress_budget(*a) == 1, pos
+    a = list(args)
+    a[18] = None                      # k_tok
+    assert L.rolesub_compress_budget(*a) == 1
+    a = list(args)
+    a[20] = big - 16                  # workspace without room for the scores
+    assert L.rolesub_compress_budget(*a) == 1
+    f32 = rsm.make_shape(1, 2, 64, 8, 6, 8, "f32")
+    p32 = rsm.Plan(f32, [[3, 2, 0, 0]], [[4, 8, 8, 8]], [1])
+    a = list(args)
+    a[0], a[1] = ctypes.byref(f32), p32.host_ptr
+    assert L.rolesub_compress_budget(*a) == 2   # the budget path is bf16, d_h = 128, S = 16 only
+    at = [ctypes.byref(shape), plan.host_ptr, fake, fake, 0, 2048, 128, fake, 0, 2048, 128, fake, fake, None,
+          fake, 0.0, fake, fake, 1 << 30, None]
+    assert L.rolesub_attend_budget(*at) == 1    # no k_tok
+    at[13] = fake
+    at[0], at[1] = ctypes.byref(f32), p32.host_ptr
+    at[5], at[6], at[9], at[10] = 1024, 64, 1024, 64
+    assert L.rolesub_attend_budget(*at) == 2
