@@ -29,8 +29,10 @@
 //   Y += P_c Z_c                   tcgen05, M=64, N=128 (rotated space)
 // Unit tail: Y / l -> bf16 smem (a staging tile of its own, so that a Q
 // slot is free as soon as its unit's last S is issued),
-// O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into the unit's Y buffer, output
-// stores.
+// O = Y R_h^T (o_q = R_h y_q, Sec. 3.2) into the unit's Y buffer; O as
+// bf16 back into the (now free) staging tile, each tail warp its own 16
+// rows, then read back and stored 16 bytes per lane, two full rows per warp
+// instruction.
 //
 // Warp roles (544 threads), all hand-offs through mbarriers. Warp w runs on
 // sub-partition w % 4.
@@ -597,8 +599,9 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         }
     } else if (warp >= 8 && warp < 12) {
         // ================= unit tail (warps 8-11) =========================
-        // y / l -> bf16 operand in the unit's Q slot; after O = Y R_h^T, the
-        // output rows. Lane quadrant w = warp % 4, same row mapping as softmax.
+        // y / l -> bf16 operand in the staging tile; after O = Y R_h^T, the
+        // output rows through the same tile. Lane quadrant w = warp % 4, same
+        // row mapping as softmax.
         const int w = warp & 3, cq = lane & 3;
         const int ra = 16 * w + (lane >> 2), rb = ra + 8;
         const uint32_t lbase = tmem + ((uint32_t)(32 * w) << 16);
@@ -640,28 +643,40 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             const bool ok = mbar_wait(B(B_OF), n & 1, status, &abort_flag, 74);
             tc_fence_after();
             __syncwarp();
-            bf16 *oa = o + ((int64_t)t.l * q_rows + t.qrow + ra) * d + (int64_t)t.h * kDh + 2 * cq;
-            bf16 *ob = oa + 8 * d;
 #pragma unroll 1
             for (int h2 = 0; h2 < 2; ++h2) {
                 uint32_t orr[32];
                 tmem_ld16x256_x8(lbase + ycol + 64u * h2, orr);
                 tmem_wait_ld();
-                if (ok) {
+                uint32_t oa8[8], ob8[8];
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const int col = 64 * h2 + 8 * j;
-                        if (ra < t.nq)
-                            *reinterpret_cast<uint32_t *>(oa + col) =
-                                pack_bf16(__uint_as_float(orr[4 * j]), __uint_as_float(orr[4 * j + 1]));
-                        if (rb < t.nq)
-                            *reinterpret_cast<uint32_t *>(ob + col) =
-                                pack_bf16(__uint_as_float(orr[4 * j + 2]), __uint_as_float(orr[4 * j + 3]));
-                    }
+                for (int j = 0; j < 8; ++j) {
+                    oa8[j] = pack_bf16(__uint_as_float(orr[4 * j]), __uint_as_float(orr[4 * j + 1]));
+                    ob8[j] = pack_bf16(__uint_as_float(orr[4 * j + 2]), __uint_as_float(orr[4 * j + 3]));
                 }
+                const uint32_t kb = yrow + 8192u * (uint32_t)h2;
+                stmatrix_x4(kb + c0, oa8[0], oa8[1], oa8[2], oa8[3]);
+                stmatrix_x4(kb + c1, oa8[4], oa8[5], oa8[6], oa8[7]);
+                stmatrix_x4(kb + 1024u + c0, ob8[0], ob8[1], ob8[2], ob8[3]);
+                stmatrix_x4(kb + 1024u + c1, ob8[4], ob8[5], ob8[6], ob8[7]);
             }
             tc_fence_before();
             mbar_arrive(B(B_OE + yb));
+            __syncwarp();
+            // this warp's 16 output rows, 16 bytes per lane and store
+            if (ok) {
+                bf16 *obase = o + ((int64_t)t.l * q_rows + t.qrow) * d + (int64_t)t.h * kDh;
+#pragma unroll
+                for (int it2 = 0; it2 < 8; ++it2) {
+                    const int i = it2 * 32 + lane, row = 16 * w + (i >> 4), c = i & 15;
+                    if (row < t.nq) {
+                        const uint4 v = ld_shared_v4(sb + kOffY + 8192u * (uint32_t)(c >> 3) + (uint32_t)row * 128u +
+                                                     ((((uint32_t)c & 7u) ^ ((uint32_t)row & 7u)) << 4));
+                        *reinterpret_cast<uint4 *>(obase + (int64_t)row * d + 8 * c) = v;
+                    }
+                }
+            }
+            __syncwarp();
             next_unit(sp, it, nu);
             ++n;
         }
