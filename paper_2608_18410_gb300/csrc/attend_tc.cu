@@ -602,7 +602,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         // y / l -> bf16 operand in the staging tile; after O = Y R_h^T, the
         // output rows through the same tile. Lane quadrant w = warp % 4, same
         // row mapping as softmax.
-        const int w = warp & 3, cq = lane & 3;
+        const int w = warp & 3;
         const int ra = 16 * w + (lane >> 2), rb = ra + 8;
         const uint32_t lbase = tmem + ((uint32_t)(32 * w) << 16);
         ChunkIt it = first;
@@ -666,7 +666,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             // this warp's 16 output rows, 16 bytes per lane and store
             if (ok) {
                 bf16 *obase = o + ((int64_t)t.l * q_rows + t.qrow) * d + (int64_t)t.h * kDh;
-#pragma unroll
+#pragma unroll 1
                 for (int it2 = 0; it2 < 8; ++it2) {
                     const int i = it2 * 32 + lane, row = 16 * w + (i >> 4), c = i & 15;
                     if (row < t.nq) {

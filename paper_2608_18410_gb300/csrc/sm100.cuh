@@ -100,12 +100,9 @@ static __device__ __noinline__ void wait_timed_out(int32_t *status, volatile int
     *abort = 1;
 }
 
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status,
-                                          volatile int *abort, int where)
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int32_t *status,
+                                                   volatile int *abort, int where)
 {
-    // a phase that has already completed costs one non-blocking test (a
-    // try_wait with a suspend hint costs several times more even then)
-    if (mbar_test(bar, parity)) return true;
     const uint64_t t0 = global_ns();
 #pragma unroll 1
     for (;;) {
@@ -115,6 +112,17 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t
     }
     wait_timed_out(status, abort, where);
     return false;
+}
+
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status,
+                                          volatile int *abort, int where)
+{
+    // a phase that has already completed costs one non-blocking test (a
+    // try_wait with a suspend hint costs several times more even then); the
+    // sleeping loop is out of line, so every wait site stays a few
+    // instructions long
+    if (mbar_test(bar, parity)) return true;
+    return mbar_wait_slow(bar, parity, status, abort, where);
 }
 
 // --------------------------------------------------------------------- TMA
