@@ -27,6 +27,9 @@ Parity status of each function (what pins it, in tests/test_oracle_pins.py):
                      K_i: counts from the allocator over pi = u . a (scipy
                      softmax), brute-force top-K_i, equal counts == the
                      fixed-k C path, every mask == dense R M R^T v attention
+  select_count / select_tokens -- Sec. 3.1 / 4.1 token reduction: the
+                     paper's 8 / 16 / 32 of 512 visual tokens, brute-force
+                     best subsets, ties and NaN scores, rows copied exactly
   compress/attend -- all-kept == dense attention (1e-10), none-kept == 0,
                      every mask on tiny inputs == dense attention over
                      R M R^T v, complement linearity, R = I textbook case,
@@ -35,6 +38,7 @@ Parity status of each function (what pins it, in tests/test_oracle_pins.py):
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import subprocess
 import threading
@@ -529,3 +533,32 @@ def attend_layer_budget(spec: Spec, q, K, packed, idx, ktok, R, scale=0.0, episo
             p /= p.sum(axis=1, keepdims=True)
             o[q0:q1, hh * s.dh:(hh + 1) * s.dh] = (p @ ztil) @ R[hh].T
     return o
+
+
+# ---------------------------------------------------------------------------
+# Token-level reduction (Sec. 3.1)
+# ---------------------------------------------------------------------------
+
+def select_count(n_view, ratio):
+    """Tokens kept per view: ceil(r * n) (Sec. 3.1), the budget split evenly
+    over the camera views (Sec. 4.1)."""
+    return int(math.ceil(float(ratio) * int(n_view)))
+
+
+def select_tokens(scores, x, ratio):
+    """scores [E][V][n], x [E][V][n][...]: per (episode, view) the k highest
+    scores (ties: lower index; NaN lowest), in token order. Returns
+    keep_idx [E][V][k] int32 and x_keep [E][V][k][...]."""
+    scores = np.asarray(scores, np.float64)
+    E, V, n = scores.shape
+    k = select_count(n, ratio)
+    keep = np.zeros((E, V, k), np.int32)
+    for e in range(E):
+        for v in range(V):
+            s = scores[e, v]
+            # plain selection by the ranking rule, one token at a time
+            order = sorted(range(n), key=lambda i: (0 if math.isnan(s[i]) else 1,
+                                                    -math.inf if math.isnan(s[i]) else s[i], -i), reverse=True)
+            keep[e, v] = np.sort(np.array(order[:k], np.int64)).astype(np.int32)
+    xk = np.take_along_axis(np.asarray(x), keep.reshape(E, V, k, *([1] * (np.asarray(x).ndim - 3))), axis=2)
+    return keep, xk

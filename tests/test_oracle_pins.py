@@ -771,3 +771,44 @@ def test_budget_forced_counts_must_meet_the_budget(oracle):
         _route_budget(oracle, p, k_force=np.array([2, 2, 1], np.int32))   # sums to 5, not 6
     with pytest.raises(ValueError):
         _route_budget(oracle, p, k_force=np.array([5, 1, 0], np.int32))   # 5 > S
+
+
+# ---------------------------------------------------------------------------
+# Token-level reduction (Sec. 3.1, Sec. 4.1)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("ratio,total", [(0.015625, 8), (0.03125, 16), (0.0625, 32)])
+def test_select_counts_match_the_papers_visual_budgets(oracle, ratio, total):
+    # Sec. 4.1: retention ratios 1/64, 1/32, 1/16 keep 8, 16, 32 of the 512
+    # visual tokens, split evenly over the two 256-token camera views
+    assert 2 * oracle.select_count(256, ratio) == total
+    assert oracle.select_count(512, ratio) == total
+
+
+def test_select_count_is_a_ceiling(oracle):
+    assert oracle.select_count(10, 0.25) == 3       # ceil(2.5)
+    assert oracle.select_count(7, 1.0) == 7
+    assert oracle.select_count(300, 0.0625) == 19   # ceil(18.75)
+
+
+def test_select_keeps_the_best_subset_brute_force(oracle):
+    rng = np.random.default_rng(50)
+    for _ in range(40):
+        n = int(rng.integers(1, 9))
+        r = float(rng.choice([0.25, 0.5, 0.75, 1.0]))
+        s = rng.standard_normal((1, 2, n))
+        x = rng.standard_normal((1, 2, n, 3))
+        keep, xk = oracle.select_tokens(s, x, r)
+        k = math.ceil(r * n)
+        for v in range(2):
+            best = max(itertools.combinations(range(n), k), key=lambda c: sum(s[0, v, list(c)]))
+            assert tuple(keep[0, v]) == tuple(sorted(best))
+            assert np.array_equal(xk[0, v], x[0, v, list(sorted(best))])
+
+
+def test_select_ties_and_nan(oracle):
+    s = np.array([[[0.5, 0.5, 0.5, 0.5]], [[np.nan, -np.inf, 0.0, -0.0]]])
+    s = s.reshape(2, 1, 4)
+    keep, _ = oracle.select_tokens(s, np.zeros((2, 1, 4, 1)), 0.5)
+    assert list(keep[0, 0]) == [0, 1]     # equal scores: lower index first
+    assert list(keep[1, 0]) == [2, 3]     # 0 and -0 tie above -inf; NaN lowest
