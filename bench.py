@@ -470,6 +470,31 @@ def run_ours(args):
     bud_c_ms = statistics.mean(a.elapsed_time(b) for a, b, c in ev_bud)
     bud_a_ms = statistics.mean(b.elapsed_time(c) for a, b, c in ev_bud)
 
+    # ---- token-level reduction (Sec. 3.1) ahead of the cache: 64 episodes x
+    # 2 camera views x 256 visual tokens, hidden d, ratio 1/16 (32 of 512) ---
+    sel_scores = torch.randn(64, 2, 256, device=dev)
+    sel_x = torch.randn(64, 2, 256, wl.d, device=dev).to(rs.tdtype)
+    sel_k = rolesub.rolesub_select_count(256, 0.0625)
+    sel_idx = torch.empty((64, 2, sel_k), dtype=torch.int32, device=dev)
+    sel_out = torch.empty((64, 2, sel_k, wl.d), dtype=rs.tdtype, device=dev)
+    for _ in range(3):
+        rolesub.rolesub_select_tokens(sel_scores, sel_x, 0.0625, sel_idx, sel_out)
+    torch.cuda.synchronize()
+    # the kept rows (17 MB) would stay in L2 between calls: flush before each
+    sel_flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    ev_sel = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(args.steps)]
+    for i in range(args.steps):
+        sel_flush.fill_(i & 0xFF)
+        ev_sel[i][0].record(stream)
+        rolesub.rolesub_select_tokens(sel_scores, sel_x, 0.0625, sel_idx, sel_out)
+        ev_sel[i][1].record(stream)
+    torch.cuda.synchronize()
+    sel_ms = statistics.mean(a.elapsed_time(b) for a, b in ev_sel)
+    del sel_flush
+    sel_bytes = 64 * 2 * (256 * 4 + sel_k * 4 + 2 * sel_k * wl.d * sel_out.element_size())
+    del sel_x
+
     # ---- end to end through the public API from pinned host buffers --------
     act = ("h", "v", "K", "q")
     host = {}
@@ -524,6 +549,9 @@ def run_ours(args):
     cab = compress_additive_bytes(wl, C_ADD)
     comp_add = {"ms": add_ms, "role_dim": C_ADD, "algorithmic_bytes": cab, "GB/s": cab / (add_ms / 1e3) / 1e9,
                 "frac": cab / (add_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
+    select = {"episodes": 64, "views": 2, "tokens_per_view": 256, "kept_per_view": sel_k, "ms": sel_ms,
+              "l2": "flushed before each call",
+              "algorithmic_bytes": sel_bytes, "GB/s": sel_bytes / (sel_ms / 1e3) / 1e9}
     budget = {"role_dim": C_ADD, "compress_ms": bud_c_ms, "compress_GB/s": cab / (bud_c_ms / 1e3) / 1e9,
               "attend_ms": bud_a_ms, "attend_GB/s": ab / (bud_a_ms / 1e3) / 1e9,
               "attend_frac": ab / (bud_a_ms / 1e3) / 1e9 / peaks["hbm_gbs"],
@@ -539,6 +567,7 @@ def run_ours(args):
                     "ms_per_step": e2e_ms},
             "gpu_launches": launches,
             "roofline": roof, "compress": comp, "compress_additive": comp_add, "budget": budget,
+            "select_tokens": select,
             "clocks": {"sm_mhz": clocks["sm_mhz"], "sm_max_mhz": clocks["sm_max_mhz"],
                        "reasons": clocks["reasons"], "samples": clocks["samples"]}}
     if ws == 1 and rank == 0 and not args.no_cpu_baseline:

@@ -301,6 +301,36 @@ rolesub_status rolesub_attend_budget(const rolesub_shape *shape, const void *pla
                                      float softmax_scale, void *o, void *workspace,
                                      size_t ws_bytes, void *stream);
 
+/*
+ * Token-level reduction (Sec. 3.1), the step before the value path: a
+ * selector scores every visual token (u_i = psi(h_i, X); the paper takes
+ * the scores from a separate method, so they are an input here) and the
+ * ceil(r |I|) highest-scoring tokens are retained, the budget divided
+ * evenly between the camera views (Sec. 4.1).
+ *
+ * rolesub_select_count: tokens kept per view, ceil(ratio * n_view) in double
+ * precision; -1 unless 0 < ratio <= 1 and n_view >= 0.
+ *
+ * rolesub_select_tokens: for each of num_episodes x num_views groups of
+ * n_view tokens (episode-major, then view; row-major rows of `hidden`
+ * elements of `dtype`), keeps the k = rolesub_select_count(n_view, ratio)
+ * tokens with the highest score (ties: lower token index; NaN scores rank
+ * lowest) in their original order.
+ *   scores   [E][V][n_view] float32 (device)
+ *   x        [E][V][n_view][hidden] (device), hidden * element size a
+ *            multiple of 16 bytes
+ * Outputs (device):
+ *   keep_idx [E][V][k] int32, the kept tokens' indices within their view,
+ *            ascending
+ *   x_keep   [E][V][k][hidden], their rows
+ * All pointers 16-byte aligned. n_view <= 16384. Errors: ROLESUB_EINVAL on
+ * bad arguments (nothing launched), ROLESUB_ECUDA on a failed launch.
+ */
+int32_t rolesub_select_count(int32_t n_view, double ratio);
+rolesub_status rolesub_select_tokens(int32_t num_episodes, int32_t num_views, int32_t n_view, double ratio,
+                                     const float *scores, const void *x, int32_t hidden, int32_t dtype,
+                                     int32_t *keep_idx, void *x_keep, void *stream);
+
 /* Waits for the stream, then reads the workspace's status word:
  * *code_out = 0 when no kernel reported bad data, else a ROLESUB_E* code.
  * *detail_out (may be NULL) receives the first reported item. */

@@ -532,6 +532,34 @@ rolesub_status rolesub_compress_budget(const rolesub_shape *shape, const void *p
     return from_cuda(rs::launch_rotate_pack(a));
 }
 
+int32_t rolesub_select_count(int32_t n_view, double ratio)
+{
+    if (n_view < 0 || !(ratio > 0.0) || ratio > 1.0) return -1;
+    const double x = ratio * (double)n_view;
+    int64_t k = (int64_t)x;
+    if ((double)k < x) ++k;   // ceil
+    return (int32_t)k;
+}
+
+rolesub_status rolesub_select_tokens(int32_t num_episodes, int32_t num_views, int32_t n_view, double ratio,
+                                     const float *scores, const void *x, int32_t hidden, int32_t dtype,
+                                     int32_t *keep_idx, void *x_keep, void *stream)
+{
+    if (num_episodes < 0 || num_views < 1 || n_view < 0 || n_view > 16384 || hidden < 1) return ROLESUB_EINVAL;
+    if (dtype != ROLESUB_F32 && dtype != ROLESUB_BF16) return ROLESUB_EINVAL;
+    const int32_t k = rolesub_select_count(n_view, ratio);
+    if (k < 0) return ROLESUB_EINVAL;
+    const int64_t row_bytes = (int64_t)hidden * elem_bytes(dtype);
+    if (row_bytes % 16 != 0) return ROLESUB_EINVAL;
+    const int64_t groups = (int64_t)num_episodes * num_views;
+    if (groups == 0 || n_view == 0) return ROLESUB_OK;
+    const void *ptrs[] = {scores, x, keep_idx, x_keep};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    return from_cuda(rs::launch_select_tokens(groups, n_view, k, scores, x, row_bytes, keep_idx, x_keep,
+                                              (cudaStream_t)stream));
+}
+
 rolesub_status rolesub_get_device_status(const void *workspace, void *stream, int32_t *code_out,
                                          int32_t *detail_out)
 {

@@ -109,6 +109,11 @@ cudaError_t launch_budget_select(const CompressArgs &a, const float *scores, uin
 cudaError_t launch_row_store_budget(const PlanView &pv, int L, const uint8_t *idx, int64_t idx_per_layer,
                                     const uint8_t *k_tok, uint4 *recs, int32_t *status, cudaStream_t stream);
 
+// Token-level reduction: per group of n scores keep the k best (ties: lower
+// index) in order, their indices and rows (row_bytes each).
+cudaError_t launch_select_tokens(int64_t groups, int n, int k, const float *scores, const void *x, int64_t row_bytes,
+                                 int32_t *keep_idx, void *x_keep, cudaStream_t stream);
+
 // Adds n to the process-wide launch counter (rolesub_launch_count).
 void count_launches(int n);
 

@@ -31,7 +31,8 @@ EXPORTS = ("rolesub_plan_size", "rolesub_layout_plan", "rolesub_workspace_size",
            "rolesub_compress", "rolesub_attend", "rolesub_get_device_status",
            "rolesub_reset_device_status", "rolesub_status_string", "rolesub_version",
            "rolesub_launch_count", "rolesub_compress_static", "rolesub_compress_additive",
-           "rolesub_budget_workspace_size", "rolesub_compress_budget", "rolesub_attend_budget")
+           "rolesub_budget_workspace_size", "rolesub_compress_budget", "rolesub_attend_budget",
+           "rolesub_select_count", "rolesub_select_tokens")
 
 STATIC_SCRATCH_BYTES = 8 << 20
 
@@ -117,10 +118,15 @@ def lib():
         L.rolesub_attend_budget.argtypes = ([sp, _vp, _vp, _vp] + [ctypes.c_int64] * 3 + [_vp]
                                             + [ctypes.c_int64] * 3 + [_vp, _vp, _vp, _vp, ctypes.c_float, _vp,
                                                                       _vp, ctypes.c_size_t, _vp])
+        L.rolesub_select_count.argtypes = [ctypes.c_int32, ctypes.c_double]
+        L.rolesub_select_count.restype = ctypes.c_int32
+        L.rolesub_select_tokens.argtypes = ([ctypes.c_int32] * 3 + [ctypes.c_double, _vp, _vp, ctypes.c_int32,
+                                                                   ctypes.c_int32, _vp, _vp, _vp])
         L.rolesub_launch_count.argtypes = []
         L.rolesub_launch_count.restype = ctypes.c_uint64
         for name in EXPORTS:
-            if name not in ("rolesub_status_string", "rolesub_version", "rolesub_launch_count"):
+            if name not in ("rolesub_status_string", "rolesub_version", "rolesub_launch_count",
+                            "rolesub_select_count"):
                 getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -264,6 +270,30 @@ def rolesub_compress_static(shape, plan: Plan, plan_dev, h, v, R, W_re, b_re, W1
         ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(h), _ptr(v), _ptr(R), _ptr(W_re),
         _ptr(b_re), _ptr(W1), _ptr(b1), _ptr(W2), _ptr(b2), float(alpha_role), float(alpha_lang),
         _ptr(packed_v), _ptr(idx), _stream(stream)))
+
+
+def rolesub_select_count(n_view, ratio):
+    return int(lib().rolesub_select_count(int(n_view), float(ratio)))
+
+
+def rolesub_select_tokens(scores, x, ratio, keep_idx=None, x_keep=None, stream=None):
+    """Token-level reduction: scores [E][V][n] float32, x [E][V][n][hidden]
+    (bf16 or float32) on the device; returns keep_idx [E][V][k] int32 and
+    x_keep [E][V][k][hidden]."""
+    import torch
+    E, V, n = scores.shape
+    hidden = x.shape[-1]
+    k = rolesub_select_count(n, ratio)
+    if k < 0:
+        raise RoleSubError("rolesub_select_count", 1)
+    if keep_idx is None:
+        keep_idx = torch.empty((E, V, max(k, 1)), dtype=torch.int32, device=x.device)
+    if x_keep is None:
+        x_keep = torch.empty((E, V, max(k, 1), hidden), dtype=x.dtype, device=x.device)
+    dt = BF16 if x.dtype == torch.bfloat16 else F32
+    _check("rolesub_select_tokens", lib().rolesub_select_tokens(
+        E, V, n, float(ratio), _ptr(scores), _ptr(x), hidden, dt, _ptr(keep_idx), _ptr(x_keep), _stream(stream)))
+    return keep_idx[:, :, :k], x_keep[:, :, :k]
 
 
 def rolesub_get_device_status(workspace, stream=None):

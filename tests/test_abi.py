@@ -228,3 +228,16 @@ def test_budget_calls_reject_bad_arguments_before_any_launch(rsm):
     at[0], at[1] = ctypes.byref(f32), p32.host_ptr
     at[5], at[6], at[9], at[10] = 1024, 64, 1024, 64
     assert L.rolesub_attend_budget(*at) == 2
+
+
+def test_select_tokens_rejects_bad_arguments_before_any_launch(rsm):
+    L = rsm.lib()
+    fake = 1 << 20
+    assert L.rolesub_select_count(256, 0.0625) == 16
+    assert L.rolesub_select_count(300, 0.0625) == 19
+    assert L.rolesub_select_count(8, 0.0) == -1
+    assert L.rolesub_select_tokens(1, 2, 8, 0.0, fake, fake, 8, 0, fake, fake, None) == 1       # ratio 0
+    assert L.rolesub_select_tokens(1, 2, 8, 0.5, fake, fake, 3, 0, fake, fake, None) == 1       # 12-byte rows
+    assert L.rolesub_select_tokens(1, 2, 8, 0.5, fake + 4, fake, 8, 0, fake, fake, None) == 1   # unaligned
+    assert L.rolesub_select_tokens(1, 2, 20000, 0.5, fake, fake, 8, 0, fake, fake, None) == 1   # n_view too big
+    assert L.rolesub_select_tokens(0, 2, 8, 0.5, None, None, 8, 0, None, None, None) == 0       # nothing to do
