@@ -4,7 +4,9 @@
 // One CTA per (128-row router tile, layer), 192 threads:
 //   warp 4  TMA producer, warp 5  MMA issuer, warps 0-3  epilogue (a
 //   thread per tile row / TMEM lane).
-// Mainloop over the hidden size d in 64-column blocks (3-stage TMA ring):
+// Mainloop over the hidden size d in 64-column blocks (4-stage TMA ring of
+// 56 KB stages; the epilogue's weights W1_a and W2 are loaded into the
+// drained ring once the last products have read it):
 //   TMEM[0,256)   += h W1_h^T      (first d input columns of W1)
 //   TMEM[256,320) += h W_re^T      (role logits)
 // Epilogue, per routed row i:
@@ -37,12 +39,15 @@ constexpr int kRows = 128;
 constexpr int kF = 256;      // router hidden
 constexpr int kC = 64;       // role dim
 constexpr int kG = 16;       // groups
-constexpr int kStages = 3;
+constexpr int kStages = 4;
 
 constexpr uint32_t kStageBytes = 16384 + 32768 + 8192;       // A | W1_h | W_re
-constexpr uint32_t kOffW1A = kStages * kStageBytes;          // 168K: W1_a [256][64]
-constexpr uint32_t kOffW2 = kOffW1A + 32768;                 // 200K: W2 [16][256]
-constexpr uint32_t kOffBar = kOffW2 + 8192;                  // 208K
+// epilogue weights go into the drained ring after the main loop, above the
+// epilogue's own operands (which use [0, 160K))
+constexpr uint32_t kOffW1A = 163840;                         // 160K: W1_a [256][64]
+constexpr uint32_t kOffW2 = kOffW1A + 32768;                 // 192K: W2 [16][256]
+constexpr uint32_t kOffBar = kStages * kStageBytes;          // 224K
+static_assert(kOffW2 + 8192 <= kOffBar, "epilogue weights inside the ring");
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
 // epilogue operands reuse the (drained) stage ring
 constexpr uint32_t kOffARhi = 0, kOffARlo = 16384, kOffUhi = 32768, kOffUlo = 98304;
@@ -78,14 +83,14 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
     const int row0 = plan.route_tiles[blockIdx.x];
     const int nkb = d / 64;
 
-    const uint32_t bar_full = sb + kOffBar;            // [3]
-    const uint32_t bar_empty = bar_full + 24;          // [3]
-    const uint32_t bar_acc = bar_full + 48, bar_w = bar_full + 56, bar_ar = bar_full + 64,
-                   bar_h = bar_full + 72, bar_u = bar_full + 80, bar_g = bar_full + 88;
+    const uint32_t bar_full = sb + kOffBar;                  // [kStages]
+    const uint32_t bar_empty = bar_full + 8 * kStages;       // [kStages]
+    const uint32_t bar_acc = bar_empty + 8 * kStages, bar_w = bar_acc + 8, bar_ar = bar_acc + 16,
+                   bar_h = bar_acc + 24, bar_u = bar_acc + 32, bar_g = bar_acc + 40;
 
     if (tid == 0) {
         abort_flag = 0;
-        for (int i = 0; i < 6; ++i) mbar_init(bar_full + 8 * i, 1);
+        for (int i = 0; i < 2 * kStages; ++i) mbar_init(bar_full + 8 * i, 1);
         mbar_init(bar_acc, 1);
         mbar_init(bar_w, 1);
         mbar_init(bar_ar, 128);
@@ -110,19 +115,30 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
             prefetch_tmap(&tm_w1);
             prefetch_tmap(&tm_wre);
             prefetch_tmap(&tm_w2);
-            // epilogue weights of this layer: W1_a (input columns d..d+C) and W2
-            mbar_expect_tx(bar_w, 32768 + 8192);
-            tma_load_3d(sb + kOffW1A, &tm_w1, d, 0, l, bar_w);
-            for (int kb = 0; kb < 4; ++kb) tma_load_3d(sb + kOffW2 + 2048 * kb, &tm_w2, 64 * kb, 0, l, bar_w);
+            bool ok = true;
             for (int kb = 0; kb < nkb; ++kb) {
                 const int s = kb % kStages;
-                if (kb >= kStages && !mbar_wait(bar_empty + 8 * s, ((kb / kStages) - 1) & 1, status, &abort_flag, 20))
+                if (kb >= kStages && !mbar_wait(bar_empty + 8 * s, ((kb / kStages) - 1) & 1, status, &abort_flag, 20)) {
+                    ok = false;
                     break;
+                }
                 const uint32_t st = sb + kStageBytes * s;
                 mbar_expect_tx(bar_full + 8 * s, kStageBytes);
                 tma_load_3d(st, &tm_h, 64 * kb, row0, l, bar_full + 8 * s);
                 tma_load_3d(st + 16384, &tm_w1, 64 * kb, 0, l, bar_full + 8 * s);
                 tma_load_3d(st + 49152, &tm_wre, 64 * kb, 0, l, bar_full + 8 * s);
+            }
+            // epilogue weights of this layer, W1_a (input columns d..d+C) and
+            // W2, into stages 2 and 3 once their last products are done
+            for (int s = 2; s < kStages && ok; ++s)
+                if (nkb > s) {
+                    const int last = s + kStages * ((nkb - 1 - s) / kStages);
+                    ok = mbar_wait(bar_empty + 8 * s, (last / kStages) & 1, status, &abort_flag, 28);
+                }
+            if (ok) {
+                mbar_expect_tx(bar_w, 32768 + 8192);
+                tma_load_3d(sb + kOffW1A, &tm_w1, d, 0, l, bar_w);
+                for (int kb = 0; kb < 4; ++kb) tma_load_3d(sb + kOffW2 + 2048 * kb, &tm_w2, 64 * kb, 0, l, bar_w);
             }
         }
     } else if (warp == 5) {
