@@ -189,3 +189,14 @@ def test_repeated_calls_are_deterministic():
     b = parity.run_gpu(wl, inp, rs=a["rs"])
     for key in ("packed", "idx", "o"):
         assert np.array_equal(a[key], b[key]), key
+
+
+@pytest.mark.parametrize("H", [1, 3, 5])
+def test_tensor_core_router_short_hidden(H):
+    """The tensor-core router (F = 256, C = 64, S = 16) with d = 128, 384 and
+    640: main loops of 2, 6 and 10 blocks, so the ring's last stages are
+    unused or partly used when the epilogue weights are loaded into them."""
+    E = synth.Episode
+    wl = synth.Workload(f"tc_router_h{H}", "bf16", L=2, H=H, dh=128, G=16, C=64, F=256,
+                        episodes=(E(140, 20, 64, 3, 6), E(9, 40, 5, 8, 16)), seed=14)
+    _run(wl, [(l, e) for l in range(2) for e in range(2)])
