@@ -249,8 +249,6 @@ int max_segment_tokens(const PlanView &pv)
 
 }  // namespace
 
-int budget_max_segment_tokens() { return 8192; }
-
 cudaError_t launch_budget_select(const CompressArgs &a, const float *scores, uint8_t *k_tok)
 {
     const rolesub_plan &P = *a.plan.hdr;
