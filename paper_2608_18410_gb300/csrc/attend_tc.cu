@@ -24,8 +24,8 @@
 //   Z_c = the chunk's kept groups scattered by index into a zero-filled
 //         64 x 128 MN-major tile. One group of d_s = 8 bf16 is one 16-byte
 //         swizzle chunk, copied by cp.async from the packed cache straight
-//         to its slot; per-row records (kept ids, packed offset) are fetched
-//         three chunks ahead.
+//         to its slot; per-row records (kept ids, packed offset) are loaded
+//         into registers two chunks ahead.
 //   Y += P_c Z_c                   tcgen05, M=64, N=128 (rotated space)
 // Unit tail: Y / l -> bf16 smem (a staging tile of its own, so that a Q
 // slot is free as soon as its unit's last S is issued),
@@ -59,9 +59,8 @@
 //   96K  R_h    32K (two 64-column K-blocks of 128 rows)
 //   128K P[3]   8K each (64 rows x 64 kv)
 //   152K Z[4]   16K each (two 64-column MN-blocks of 64 kv rows)
-//   216K records 4 x 1K
-//   220K row sums 2 x 64 fp32 (softmax -> unit tail)
-//   then the unit list and the barriers
+//   216K row sums 2 x 64 fp32 (softmax -> unit tail)
+//   217K the unit list (up to 512 units per CTA and launch), the barriers
 // TMEM (448 of 512 columns): S[3] at 0, 64 and 128, Y[2] at 192 and 320
 // (each later holding its unit's O).
 #include <cuda.h>
@@ -84,7 +83,7 @@ constexpr int kChunk = 64;   // cache tokens per chunk
 constexpr int kQRows = 64;   // query rows per unit
 constexpr int kDh = 128;
 constexpr int kG = 16;       // groups per head (d_s = 8)
-constexpr int kMaxUnits = 256;   // units per CTA and launch (unit list in smem)
+constexpr int kMaxUnits = 512;   // units per CTA and launch (unit list in smem)
 constexpr int kKSlots = 3;
 constexpr float kRescaleLog2 = 8.f;   // raise the reference max beyond 2^8 growth
 
@@ -96,8 +95,7 @@ constexpr int kSBufs = 3;                             // S (TMEM) and P (smem) b
 constexpr uint32_t kOffP = 131072;                    // 3 x 8K
 constexpr uint32_t kOffZ = kOffP + kSBufs * 8192;     // 4 x 16K ring
 constexpr int kZSlots = 4;
-constexpr uint32_t kOffRec = kOffZ + kZSlots * 16384; // 4 x 64 x 16 B
-constexpr uint32_t kOffL = kOffRec + 4096;           // 2 x 64 fp32 row sums
+constexpr uint32_t kOffL = kOffZ + kZSlots * 16384;   // 2 x 64 fp32 row sums
 constexpr uint32_t kOffUnits = kOffL + 1024;         // kMaxUnits x 16 B unit records
 constexpr uint32_t kOffBar = kOffUnits + 16 * kMaxUnits;
 constexpr uint32_t kSmemBytes = kOffBar + 512 + 1024;
@@ -414,40 +412,40 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         }
     } else if (warp == 4 || warp == 5 || warp == 12 || warp == 13) {
         // ================= value gather (one kv row per thread) ===========
-        // Two gatherers of 64 threads (warps 4-5 and 12-13) take the even and
-        // the odd chunks. Chunk g goes to Z slot g % 4; its row record is
-        // fetched one own chunk (two chunks) ahead. At chunk g a gatherer
-        // publishes its previous chunk g - 2 (copies complete), waits for
+        // Three gatherers of 64 threads (warps 4-5, 12-13, 17-18) take chunks
+        // g = 0, 1, 2 mod 3. Chunk g goes to Z slot g % 4; its row record is
+        // loaded into registers one own chunk ahead. At chunk g a gatherer
+        // publishes its previous chunk g - 3 (copies complete), waits for
         // the product of chunk g - 4 to free the slot, copies the kept
         // groups of chunk g by cp.async straight into their swizzled slots of
         // the tile and zeroes the groups left over from the slot's previous
         // chunk.
-        const int par = warp >= 12 ? 1 : 0, jl = tid & 63;   // warps 12-13: odd chunks
+        const int par = (warp == 4 || warp == 5) ? 0 : 1;
+        const int jl = ((warp & 1) ? 32 : 0) + lane;
         const uint32_t sw = (uint32_t)(jl & 7);
         // groups of this thread's row that may be non-zero, per Z slot (16 bits
         // each); a slot's first use clears everything
         uint64_t dirty = ~0ull;
         ChunkIt it = first;
         uint32_t g = 0;
-        if (par == 1) {
-            it_next(sp, it, nu);
-            g = 1;
-        }
+        for (int p = 0; p < par; ++p) it_next(sp, it, nu);
+        g = (uint32_t)par;
         ChunkIt ahead = it;
-        auto stage_rec = [&](uint32_t gg) {   // record of chunk gg (= ahead), then ahead += 2
+        uint4 mnext = make_uint4(0, 0, 0, 0);
+        auto fetch_rec = [&]() {   // record of chunk `ahead`, then ahead += 3
+            mnext = make_uint4(0, 0, 0, 0);
             if (ahead.k < nu) {
                 const int r = ahead.c * kChunk + jl;
-                if (r < ahead.t.nc)
-                    cp_async16(sb + kOffRec + (gg & 3u) * 1024u + (uint32_t)jl * 16u,
-                               rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
+                if (r < ahead.t.nc) mnext = __ldg(rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
             }
             it_next(sp, ahead, nu);
             it_next(sp, ahead, nu);
-            cp_async_commit();
         };
-        stage_rec(g);
+        fetch_rec();
         for (; it.k < nu && !abort_flag; g += 2) {
-            cp_async_wait_group<0>();   // record g and the copies of chunk g - 2 have landed
+            const uint4 m = mnext;
+            fetch_rec();
+            cp_async_wait_group<0>();   // the copies of chunk g - 3 have landed
             if (g >= 2) {
                 fence_async_smem();
                 mbar_arrive(B(B_ZF + ((g - 2) & 3u)));
@@ -458,7 +456,6 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             uint32_t kept = 0;
             const uint32_t zrow = sb + kOffZ + 16384u * (g & 3u) + (uint32_t)jl * 128u;
             if (jl < nk) {
-                const uint4 m = *reinterpret_cast<const uint4 *>(sp + kOffRec + (g & 3u) * 1024u + (uint32_t)jl * 16u);
                 const int k = (int)(m.w >> 27);
                 const uint64_t gid = (uint64_t)m.x | ((uint64_t)m.y << 32);
                 const bf16 *src = packed + (int64_t)it.t.l * packed_per_layer +
@@ -475,7 +472,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
                 st_shared_v4(zrow + (gg >> 3) * 8192u + (((gg & 7u) ^ sw) << 4), 0, 0, 0, 0);
             }
             dirty = (dirty & ~(0xFFFFull << sh)) | ((uint64_t)kept << sh);
-            stage_rec(g + 2);   // also commits this chunk's copies
+            cp_async_commit();
             it_next(sp, it, nu);
             it_next(sp, it, nu);
         }
