@@ -230,23 +230,24 @@ def alloc_inputs(wl: Workload):
     }
 
 
-def _fill_layer_weights(wl, out, layer):
+def _fill_layer_weights(wl, out, layer, slot=None):
+    slot = layer if slot is None else slot
     s, d = wl.seed, wl.d
     R = np.empty((wl.H, wl.dh, wl.dh), np.float64)
     rng = _rng(s, layer, 0, TID["R"])
     for hh in range(wl.H):
         R[hh] = haar_orthogonal(rng, wl.dh)
-    out["R"][layer] = _store(R.astype(np.float32), wl.dtype)
-    out["W_re"][layer] = _store(_normal(s, layer, 0, TID["W_re"], (wl.C, d), 0.02), wl.dtype)
-    out["b_re"][layer] = _normal(s, layer, 0, TID["b_re"], (wl.C,), 0.02)
-    out["W1"][layer] = _store(_normal(s, layer, 0, TID["W1"], (wl.F, 2 * d + wl.C), 0.02), wl.dtype)
-    out["b1"][layer] = _normal(s, layer, 0, TID["b1"], (wl.F,), 0.02)
+    out["R"][slot] = _store(R.astype(np.float32), wl.dtype)
+    out["W_re"][slot] = _store(_normal(s, layer, 0, TID["W_re"], (wl.C, d), 0.02), wl.dtype)
+    out["b_re"][slot] = _normal(s, layer, 0, TID["b_re"], (wl.C,), 0.02)
+    out["W1"][slot] = _store(_normal(s, layer, 0, TID["W1"], (wl.F, 2 * d + wl.C), 0.02), wl.dtype)
+    out["b1"][slot] = _normal(s, layer, 0, TID["b1"], (wl.F,), 0.02)
     W2 = _normal(s, layer, 0, TID["W2"], (wl.G, wl.F), 0.02)
     b2 = _normal(s, layer, 0, TID["b2"], (wl.G,), 0.02)
     if wl.near_tie:
         W2, b2 = _near_tie_rows(wl, layer, W2, b2)
-    out["W2"][layer] = _store(W2, wl.dtype)
-    out["b2"][layer] = b2
+    out["W2"][slot] = _store(W2, wl.dtype)
+    out["b2"][slot] = b2
 
 
 def _near_tie_rows(wl, layer, W2, b2):
@@ -283,6 +284,32 @@ def _fill_layer_acts(wl, out, layer):
                 _normal(s, layer, e, TID["q"], (ep.n_query, d)), wl.dtype)
         r += n
         qrow += ep.n_query
+
+
+def gen_layer_weights(wl: Workload, layer: int):
+    """The weights of one layer, the same draws as gen_inputs makes for it."""
+    sd = storage_dtype(wl.dtype)
+    d = wl.d
+    out = {"R": np.empty((1, wl.H, wl.dh, wl.dh), sd), "W_re": np.empty((1, wl.C, d), sd),
+           "b_re": np.empty((1, wl.C), np.float32), "W1": np.empty((1, wl.F, 2 * d + wl.C), sd),
+           "b1": np.empty((1, wl.F), np.float32), "W2": np.empty((1, wl.G, wl.F), sd),
+           "b2": np.empty((1, wl.G), np.float32)}
+    _fill_layer_weights(wl, out, layer, slot=0)
+    return {k: v[0] for k, v in out.items()}
+
+
+def gen_episode_acts(wl: Workload, layer: int, e: int):
+    """h, v, K [n_cache][d] and q [n_query][d] of one episode of one layer,
+    the same draws as gen_inputs makes for it."""
+    s, d = wl.seed, wl.d
+    ep = wl.episodes[e]
+    out = {}
+    for name in ("h", "v", "K"):
+        out[name] = _store(_normal(s, layer, e, TID[name], (ep.n_cache, d)), wl.dtype) if ep.n_cache else \
+            np.empty((0, d), storage_dtype(wl.dtype))
+    out["q"] = _store(_normal(s, layer, e, TID["q"], (ep.n_query, d)), wl.dtype) if ep.n_query else \
+        np.empty((0, d), storage_dtype(wl.dtype))
+    return out
 
 
 def gen_inputs(wl: Workload, threads: int = 8):
