@@ -412,14 +412,14 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         }
     } else if (warp == 4 || warp == 5 || warp == 12 || warp == 13) {
         // ================= value gather (one kv row per thread) ===========
-        // Three gatherers of 64 threads (warps 4-5, 12-13, 17-18) take chunks
-        // g = 0, 1, 2 mod 3. Chunk g goes to Z slot g % 4; its row record is
-        // loaded into registers one own chunk ahead. At chunk g a gatherer
-        // publishes its previous chunk g - 3 (copies complete), waits for
-        // the product of chunk g - 4 to free the slot, copies the kept
-        // groups of chunk g by cp.async straight into their swizzled slots of
-        // the tile and zeroes the groups left over from the slot's previous
-        // chunk.
+        // Two gatherers of 64 threads (warps 4-5 and 12-13) take the even and
+        // the odd chunks. Chunk g goes to Z slot g % 4; its row record is
+        // loaded into registers one own chunk (two chunks) ahead. At chunk g
+        // a gatherer publishes its previous chunk g - 2 (copies complete),
+        // waits for the product of chunk g - 4 to free the slot, copies the
+        // kept groups of chunk g by cp.async straight into their swizzled
+        // slots of the tile and zeroes the groups left over from the slot's
+        // previous chunk.
         const int par = (warp == 4 || warp == 5) ? 0 : 1;
         const int jl = ((warp & 1) ? 32 : 0) + lane;
         const uint32_t sw = (uint32_t)(jl & 7);
@@ -427,12 +427,11 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         // each); a slot's first use clears everything
         uint64_t dirty = ~0ull;
         ChunkIt it = first;
-        uint32_t g = 0;
-        for (int p = 0; p < par; ++p) it_next(sp, it, nu);
-        g = (uint32_t)par;
+        uint32_t g = (uint32_t)par;
+        if (par) it_next(sp, it, nu);
         ChunkIt ahead = it;
         uint4 mnext = make_uint4(0, 0, 0, 0);
-        auto fetch_rec = [&]() {   // record of chunk `ahead`, then ahead += 3
+        auto fetch_rec = [&]() {   // record of chunk `ahead`, then ahead += 2
             mnext = make_uint4(0, 0, 0, 0);
             if (ahead.k < nu) {
                 const int r = ahead.c * kChunk + jl;
@@ -445,7 +444,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         for (; it.k < nu && !abort_flag; g += 2) {
             const uint4 m = mnext;
             fetch_rec();
-            cp_async_wait_group<0>();   // the copies of chunk g - 3 have landed
+            cp_async_wait_group<0>();   // the copies of chunk g - 2 have landed
             if (g >= 2) {
                 fence_async_smem();
                 mbar_arrive(B(B_ZF + ((g - 2) & 3u)));
