@@ -556,6 +556,48 @@ def run_ours(args):
     sel_bytes = 64 * 2 * (256 * 4 + sel_k * 4 + 2 * sel_k * wl.d * sel_out.element_size())
     del sel_x
 
+    # ---- one OpenVLA-OFT layer (c1), a launch-latency-bound step: eager
+    # calls and the same step replayed from a CUDA graph, L2 flushed --------
+    wl1 = synth.c1()
+    inp1 = synth.gen_inputs(wl1)
+    rs1 = rolesub.RoleSub(wl1.L, wl1.H, wl1.dh, wl1.G, wl1.C, wl1.F, wl1.dtype, wl1.n_tok_array(),
+                          wl1.k_array(), wl1.n_query_array(), device=dev)
+    d1 = {k: to_dev(v) for k, v in inp1.items()}
+    p1, i1 = rs1.new_outputs()
+    o1 = torch.empty((wl1.L, wl1.q_rows, wl1.d), dtype=rs1.tdtype, device=dev)
+    lat_flush = torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def step1():
+        rs1.compress(d1["h"], d1["v"], d1["R"], d1["W_re"], d1["b_re"], d1["W1"], d1["b1"], d1["W2"], d1["b2"],
+                     wl1.alpha_role, wl1.alpha_lang, packed=p1, idx=i1)
+        rs1.attend(d1["q"], d1["K"], p1, i1, d1["R"], o=o1)
+
+    gstream = torch.cuda.Stream()
+    gstream.wait_stream(stream)
+    with torch.cuda.stream(gstream):
+        for _ in range(3):
+            step1()
+    stream.wait_stream(gstream)
+    torch.cuda.synchronize()
+    graph1 = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph1):
+        step1()
+
+    def time_latency(fn):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+        for i in range(args.steps):
+            lat_flush.fill_(i & 0xFF)
+            evs[i][0].record(stream)
+            fn()
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
+
+    lat_eager = time_latency(step1)
+    lat_graph = time_latency(graph1.replay)
+    del lat_flush, graph1
+
     # ---- end to end through the public API from pinned host buffers --------
     act = ("h", "v", "K", "q")
     host = {}
@@ -610,6 +652,8 @@ def run_ours(args):
     cab = compress_additive_bytes(wl, C_ADD)
     comp_add = {"ms": add_ms, "role_dim": C_ADD, "algorithmic_bytes": cab, "GB/s": cab / (add_ms / 1e3) / 1e9,
                 "frac": cab / (add_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
+    latency = {"workload": wl1.name, "l2": "flushed before each step", "eager_ms": lat_eager,
+               "graph_ms": lat_graph, "query_tokens_per_s_per_layer_graph": wl1.q_rows / (lat_graph / 1e3)}
     select = {"episodes": 64, "views": 2, "tokens_per_view": 256, "kept_per_view": sel_k, "ms": sel_ms,
               "l2": "flushed before each call",
               "algorithmic_bytes": sel_bytes, "GB/s": sel_bytes / (sel_ms / 1e3) / 1e9}
@@ -628,7 +672,7 @@ def run_ours(args):
                     "ms_per_step": e2e_ms},
             "gpu_launches": launches,
             "roofline": roof, "compress": comp, "compress_additive": comp_add, "budget": budget,
-            "select_tokens": select,
+            "select_tokens": select, "latency_one_layer": latency,
             "clocks": {"sm_mhz": clocks["sm_mhz"], "sm_max_mhz": clocks["sm_max_mhz"],
                        "reasons": clocks["reasons"], "samples": clocks["samples"]}}
     if ws == 1 and rank == 0 and not args.no_cpu_baseline:
