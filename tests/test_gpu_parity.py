@@ -200,3 +200,13 @@ def test_tensor_core_router_short_hidden(H):
     wl = synth.Workload(f"tc_router_h{H}", "bf16", L=2, H=H, dh=128, G=16, C=64, F=256,
                         episodes=(E(140, 20, 64, 3, 6), E(9, 40, 5, 8, 16)), seed=14)
     _run(wl, [(l, e) for l in range(2) for e in range(2)])
+
+
+def test_attention_split_over_launches():
+    """More units than one launch holds (512 per CTA): 320 tiny episodes x 32
+    heads x 8 layers = 81,920 units, so the call runs two launches; sampled
+    pairs sit in both."""
+    E = synth.Episode
+    eps = [E(8 + (i % 5), 4 + (i % 3), 1 + (i % 2), 2 + (i % 3), 4) for i in range(320)]
+    wl = synth.Workload("many_units", "bf16", L=8, H=32, dh=128, G=16, C=8, F=32, episodes=tuple(eps), seed=15)
+    _run(wl, [(0, 0), (0, 319), (3, 160), (7, 1), (7, 318)])
