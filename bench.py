@@ -337,7 +337,10 @@ def oracle_sample_all_cores(wl, key, layers, budget_s=10.0, pool=None, cores=Non
     order = [(l, e) for l in range(wl.L) for e in range(wl.E)]
     rng = np.random.default_rng(seed)
     rng.shuffle(order)
-    jobs = [(key, layers, w, [tuple(map(int, x)) for x in order[w::cores]], budget_s) for w in range(cores)]
+    # each process's random share, grouped by layer so that it draws each
+    # layer's weights once
+    jobs = [(key, layers, w, sorted((tuple(map(int, x)) for x in order[w::cores]), key=lambda t: t[0]), budget_s)
+            for w in range(cores)]
     if pool is None:
         with mp.get_context("spawn").Pool(cores) as p:
             res = p.map(_oracle_worker, jobs)
@@ -357,7 +360,8 @@ def run_reference(args):
         return 0
     import multiprocessing as mp
     wl = make_workload(args.workload, 0, args.layers)
-    per_step_budget = max(1.0, min(15.0, 150.0 / max(1, args.steps + args.warmup)))
+    # about a minute of oracle work over the steps (plus input generation)
+    per_step_budget = max(0.5, min(15.0, 60.0 / max(1, args.steps + args.warmup)))
     cores = os.cpu_count() or 1
     vals = []
     meas = None
