@@ -30,6 +30,11 @@ Parity status of each function (what pins it, in tests/test_oracle_pins.py):
   select_count / select_tokens -- Sec. 3.1 / 4.1 token reduction: the
                      paper's 8 / 16 / 32 of 512 visual tokens, brute-force
                      best subsets, ties and NaN scores, rows copied exactly
+  pack_layer_dense / attend_layer_dense -- one dense d x d R (Sec. 4.1):
+                     all kept == dense attention, none kept == 0, every mask
+                     == dense attention over explicit R M R^T v, and the
+                     per-head C oracle reproduced exactly by the dense R
+                     blockdiag(R_h) with the head-interleaving permutation
   compress/attend -- all-kept == dense attention (1e-10), none-kept == 0,
                      every mask on tiny inputs == dense attention over
                      R M R^T v, complement linearity, R = I textbook case,
@@ -562,3 +567,75 @@ def select_tokens(scores, x, ratio):
             keep[e, v] = np.sort(np.array(order[:k], np.int64)).astype(np.int32)
     xk = np.take_along_axis(np.asarray(x), keep.reshape(E, V, k, *([1] * (np.asarray(x).ndim - 3))), axis=2)
     return keep, xk
+
+
+# ---------------------------------------------------------------------------
+# Dense rotation (Sec. 4.1 geometry: one d x d orthonormal R per layer, S
+# contiguous groups of d / S rotated dimensions)
+# ---------------------------------------------------------------------------
+
+def pack_layer_dense(spec: Spec, v, Rd, idx, episodes=None):
+    """Sec. 3.2 with one dense R: z_i = R^T v_i over all d = H d_h dims, split
+    into S contiguous groups of g = d / S; segment (n tokens, k) holds
+    [n][k][g] values (the kept groups in index order). Returns packed
+    [packed_elems] float64."""
+    s = spec
+    lay = s.lay
+    g = s.d // s.G
+    packed = np.zeros(max(lay["packed_elems"], 1))
+    nt = s.n_tok.reshape(-1)
+    kt = s.k.reshape(-1)
+    Rd = np.asarray(Rd, np.float64)
+    for e in (range(s.E) if episodes is None else episodes):
+        for m in range(4):
+            sgi = 4 * e + m
+            n, k, r0 = int(nt[sgi]), int(kt[sgi]), int(lay["row_off"][sgi])
+            if n == 0 or k == 0:
+                continue
+            io, po = int(lay["idx_off"][sgi]), int(lay["packed_off"][sgi])
+            z = np.asarray(v[r0:r0 + n], np.float64) @ Rd          # rows: z = R^T v
+            for i in range(n):
+                for j in range(k):
+                    grp = int(idx[io + i * k + j])
+                    dst = po + (i * k + j) * g
+                    packed[dst:dst + g] = z[i, grp * g:(grp + 1) * g]
+    return packed[:lay["packed_elems"]]
+
+
+def attend_layer_dense(spec: Spec, q, K, packed, idx, Rd, scale=0.0, episodes=None):
+    """Attention over a dense-R cache (Sec. 3): per head h,
+    p = softmax_j(q_h . k_{j,h} * scale), y = sum_j p_j M_j z_j (all d rotated
+    dims, zeros outside the kept groups), o_h = R[rows of head h] y.
+    Returns o [q_rows][d] float64."""
+    s = spec
+    lay = s.lay
+    g = s.d // s.G
+    sc = scale if scale > 0 else 1.0 / np.sqrt(s.dh)
+    o = np.zeros((int(s.ep_q[-1]), s.d))
+    nt = s.n_tok.reshape(-1)
+    kt = s.k.reshape(-1)
+    Rd = np.asarray(Rd, np.float64)
+    for e in (range(s.E) if episodes is None else episodes):
+        r0, r1 = int(s.ep_row[e]), int(s.ep_row[e + 1])
+        q0, q1 = int(s.ep_q[e]), int(s.ep_q[e + 1])
+        if q1 == q0 or r1 == r0:
+            continue
+        zm = np.zeros((r1 - r0, s.d))          # M_j z_j of every cache token
+        for m in range(4):
+            sgi = 4 * e + m
+            n, k, rs_ = int(nt[sgi]), int(kt[sgi]), int(lay["row_off"][sgi])
+            io, po = int(lay["idx_off"][sgi]), int(lay["packed_off"][sgi])
+            for i in range(n):
+                for j in range(k):
+                    grp = int(idx[io + i * k + j])
+                    src = po + (i * k + j) * g
+                    zm[rs_ - r0 + i, grp * g:(grp + 1) * g] = packed[src:src + g]
+        for hh in range(s.H):
+            qh = np.asarray(q[q0:q1, hh * s.dh:(hh + 1) * s.dh], np.float64)
+            kh = np.asarray(K[r0:r1, hh * s.dh:(hh + 1) * s.dh], np.float64)
+            sco = qh @ kh.T * sc
+            sco -= sco.max(axis=1, keepdims=True)
+            p = np.exp(sco)
+            p /= p.sum(axis=1, keepdims=True)
+            o[q0:q1, hh * s.dh:(hh + 1) * s.dh] = (p @ zm) @ Rd[hh * s.dh:(hh + 1) * s.dh, :].T
+    return o

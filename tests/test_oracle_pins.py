@@ -812,3 +812,83 @@ def test_select_ties_and_nan(oracle):
     keep, _ = oracle.select_tokens(s, np.zeros((2, 1, 4, 1)), 0.5)
     assert list(keep[0, 0]) == [0, 1]     # equal scores: lower index first
     assert list(keep[1, 0]) == [2, 3]     # 0 and -0 tie above -inf; NaN lowest
+
+
+# ---------------------------------------------------------------------------
+# Dense rotation (one d x d R, S contiguous groups of d / S dims; Sec. 4.1)
+# ---------------------------------------------------------------------------
+
+def _dense_run(oracle, p, Rd, idx_force):
+    spec = oracle.Spec(p["H"], p["dh"], p["G"], p["C"], p["F"], p["n_tok"], p["k"], p["n_q"])
+    packed = oracle.pack_layer_dense(spec, p["v"], Rd, idx_force)
+    return spec, packed, oracle.attend_layer_dense(spec, p["q"], p["K"], packed, idx_force, Rd)
+
+
+def _all_idx(n_rows, G, k):
+    return np.tile(np.arange(k, dtype=np.uint8) if k < G else np.arange(G, dtype=np.uint8), n_rows)
+
+
+def test_dense_all_groups_kept_equals_dense_attention(oracle):
+    rng = np.random.default_rng(70)
+    H, dh, G = 2, 8, 4
+    p = rnd_problem(rng, H=H, dh=dh, G=G, n_tok=((5, 3, 0, 0),), k=((G, G, G, G),), n_q=(4,))
+    Rd = haar(rng, H * dh)
+    _, _, o = _dense_run(oracle, p, Rd, _all_idx(8, G, G))
+    assert rel_err(o, dense_attention(p), dh) < 1e-10      # R M R^T v = v when every group is kept
+
+
+def test_dense_no_groups_kept_gives_zero(oracle):
+    rng = np.random.default_rng(71)
+    p = rnd_problem(rng, H=2, dh=8, G=4, n_tok=((5, 3, 0, 0),), k=((0, 0, 4, 4),), n_q=(4,))
+    _, _, o = _dense_run(oracle, p, haar(rng, 16), np.zeros(0, np.uint8))
+    assert np.all(o == 0)
+
+
+def test_dense_every_mask_equals_attention_over_explicit_routed_values(oracle):
+    rng = np.random.default_rng(72)
+    H, dh, G = 2, 4, 4
+    d, gw = H * dh, H * dh // G
+    for k in (1, 2, 3):
+        p = rnd_problem(rng, H=H, dh=dh, G=G, n_tok=((3, 0, 0, 0),), k=((k, G, G, G),), n_q=(2,))
+        Rd = haar(rng, d)
+        subsets = list(itertools.combinations(range(G), k))
+        for masks in itertools.product(subsets, repeat=3):
+            fx = np.array([g for m in masks for g in m], np.uint8)
+            _, _, o = _dense_run(oracle, p, Rd, fx)
+            vt = []
+            for r in range(3):
+                mvec = np.zeros(d)
+                for g in masks[r]:
+                    mvec[g * gw:(g + 1) * gw] = 1.0
+                vt.append(Rd @ np.diag(mvec) @ Rd.T @ p["v"][r])   # v~ = R M R^T v, all heads at once
+            vt = np.array(vt)
+            ref = dense_attention(p, lambda e, h, r0, r1: vt[r0:r1, h * dh:(h + 1) * dh])
+            assert np.max(np.abs(o - ref)) <= 1e-12, (k, masks)
+
+
+def test_dense_block_diagonal_rotation_reproduces_the_per_head_oracle(oracle):
+    # R = blockdiag(R_1 .. R_H) with the permutation that makes dense group s
+    # the s-th group of every head: the dense restatement (numpy) must give
+    # the per-head C oracle's values and outputs exactly
+    rng = np.random.default_rng(73)
+    H, dh, G = 3, 8, 4
+    ds, d = dh // G, H * dh
+    p = rnd_problem(rng, H=H, dh=dh, G=G, n_tok=((6, 4, 0, 0),), k=((2, 3, G, G),), n_q=(3,))
+    spec, c, o_head = run(oracle, p)
+    B = np.zeros((d, d))
+    for hh in range(H):
+        B[hh * dh:(hh + 1) * dh, hh * dh:(hh + 1) * dh] = p["R"][hh]
+    perm = np.zeros(d, np.int64)     # dense coordinate -> per-head coordinate
+    for s_ in range(G):
+        for hh in range(H):
+            for t in range(ds):
+                perm[s_ * H * ds + hh * ds + t] = hh * dh + s_ * ds + t
+    Rd = B[:, perm]
+    packed = oracle.pack_layer_dense(spec, p["v"], Rd, c["idx"])
+    o_dense = oracle.attend_layer_dense(spec, p["q"], p["K"], packed, c["idx"], Rd)
+    assert np.max(np.abs(o_dense - o_head)) < 1e-12
+    lay = spec.lay
+    for m, (n, k) in enumerate(((6, 2), (4, 3))):
+        a = packed[lay["packed_off"][m]: lay["packed_off"][m] + n * k * H * ds].reshape(n, k, H, ds)
+        b = c["packed"][lay["packed_off"][m]: lay["packed_off"][m] + H * n * k * ds].reshape(H, n, k, ds)
+        assert np.max(np.abs(a - b.transpose(1, 2, 0, 3))) < 1e-12
