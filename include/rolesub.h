@@ -331,6 +331,44 @@ rolesub_status rolesub_select_tokens(int32_t num_episodes, int32_t num_views, in
                                      const float *scores, const void *x, int32_t hidden, int32_t dtype,
                                      int32_t *keep_idx, void *x_keep, void *stream);
 
+/*
+ * The dense-rotation geometry of the paper's setup (Sec. 4.1): one d x d
+ * orthonormal R per layer (d = H d_h) and S contiguous groups of g = d / S
+ * rotated dims, in place of the per-head R_h of rolesub_compress.
+ *
+ * rolesub_compress_dense: routing as rolesub_compress (same router, same
+ * indices), then z_i = R^T v_i over all d dims and the kept groups packed:
+ * segment (n tokens, k) holds [n][k][g] values, token i's groups in index
+ * order at packed_off + (i k + j) g (the plan's segment sizes are the same:
+ * n k H d_s = n k g).
+ *   R_dense [L][d][d] (R[m][n], dtype); other arguments as rolesub_compress.
+ * rolesub_attend_dense: attention over such a cache; every head's output
+ * needs all d rotated dims (o_{q,h} = R_h sum_j p_j M_j z_j with R_h the d_h
+ * rows of head h), so the call first forms the routed values
+ * v~_j = R M_j z_j of every cache row on the tensor core and then attends
+ * over them; arguments as rolesub_attend plus R_dense.
+ * workspace: at least rolesub_dense_workspace_size bytes for either call
+ * (the common workspace, then 2 L rows d + L H d_h^2 bf16 elements).
+ * Supported geometry: bf16, d_h = 128, S = 16, d a multiple of 256;
+ * otherwise ROLESUB_EUNSUPPORTED.
+ */
+rolesub_status rolesub_dense_workspace_size(const rolesub_shape *shape, const void *plan_host,
+                                            size_t *bytes);
+rolesub_status rolesub_compress_dense(const rolesub_shape *shape, const void *plan_host,
+                                      const void *plan_dev, const void *h, const void *v,
+                                      const void *R_dense, const void *W_re, const float *b_re,
+                                      const void *W1, const float *b1, const void *W2,
+                                      const float *b2, float alpha_role, float alpha_lang,
+                                      void *packed_v, uint8_t *idx, void *workspace,
+                                      size_t ws_bytes, void *stream);
+rolesub_status rolesub_attend_dense(const rolesub_shape *shape, const void *plan_host,
+                                    const void *plan_dev, const void *q, int64_t q_layer_stride,
+                                    int64_t q_row_stride, int64_t q_head_stride, const void *K,
+                                    int64_t k_layer_stride, int64_t k_row_stride,
+                                    int64_t k_head_stride, const void *packed_v,
+                                    const uint8_t *idx, const void *R_dense, float softmax_scale,
+                                    void *o, void *workspace, size_t ws_bytes, void *stream);
+
 /* Waits for the stream, then reads the workspace's status word:
  * *code_out = 0 when no kernel reported bad data, else a ROLESUB_E* code.
  * *detail_out (may be NULL) receives the first reported item. */

@@ -134,6 +134,24 @@ Workspace carve(const WsSizes &w, void *base)
 
 rolesub_status from_cuda(cudaError_t e) { return e == cudaSuccess ? ROLESUB_OK : ROLESUB_ECUDA; }
 
+// The dense-rotation path: bf16, d_h = 128, S = 16 (the tensor-core
+// rotation's store records and the tensor-core attention), d % 256 == 0 (the
+// GEMM's column tile).
+bool dense_supported(const rolesub_shape *s)
+{
+    const int d = s->num_heads * s->head_dim;
+    return rs::rotate_tc_supported(s) && rs::attend_tc_supported(s) && d % 256 == 0 && d <= 65536;
+}
+
+// Z (compress) or M z and v~ (attend), [L][rows][d] bf16 each, and the
+// identity rotations [L][H][d_h][d_h] bf16, after the common workspace.
+size_t dense_extra_bytes(const rolesub_shape *s, const rolesub_plan *p)
+{
+    const size_t d = (size_t)s->num_heads * s->head_dim, L = s->num_layers;
+    const size_t vals = align_up(2 * L * (size_t)p->rows_per_layer * d, kAlign);
+    return 2 * vals + align_up(2 * L * s->num_heads * (size_t)s->head_dim * s->head_dim, kAlign);
+}
+
 bool budget_supported(const rolesub_shape *s, const PlanView &pv)
 {
     if (!rs::rotate_tc_supported(s) || !rs::attend_tc_supported(s) || !rs::additive_tc_supported(s)) return false;
@@ -558,6 +576,132 @@ rolesub_status rolesub_select_tokens(int32_t num_episodes, int32_t num_views, in
         if (!p || !aligned16(p)) return ROLESUB_EINVAL;
     return from_cuda(rs::launch_select_tokens(groups, n_view, k, scores, x, row_bytes, keep_idx, x_keep,
                                               (cudaStream_t)stream));
+}
+
+rolesub_status rolesub_dense_workspace_size(const rolesub_shape *shape, const void *plan_host, size_t *bytes)
+{
+    if (!shape_ok(shape) || !bytes) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, nullptr, &pv);
+    if (st != ROLESUB_OK) return st;
+    *bytes = ws_sizes(shape, pv.hdr).total + dense_extra_bytes(shape, pv.hdr);
+    return ROLESUB_OK;
+}
+
+rolesub_status rolesub_compress_dense(const rolesub_shape *shape, const void *plan_host, const void *plan_dev,
+                                      const void *h, const void *v, const void *R_dense, const void *W_re,
+                                      const float *b_re, const void *W1, const float *b1, const void *W2,
+                                      const float *b2, float alpha_role, float alpha_lang, void *packed_v,
+                                      uint8_t *idx, void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!shape_ok(shape)) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, plan_dev, &pv);
+    if (st != ROLESUB_OK) return st;
+    if (!plan_dev) return ROLESUB_EINVAL;
+    const void *ptrs[] = {h, v, R_dense, W_re, b_re, W1, b1, W2, b2, workspace};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    const rolesub_plan &P = *pv.hdr;
+    if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
+    if (P.idx_bytes_per_layer > 0 && (!idx || !aligned16(idx))) return ROLESUB_EINVAL;
+    if (!isfinite(alpha_role) || !isfinite(alpha_lang)) return ROLESUB_EINVAL;
+    if (!dense_supported(shape) || !rs::router_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    const WsSizes w = ws_sizes(shape, pv.hdr);
+    if (ws_bytes < w.total + dense_extra_bytes(shape, pv.hdr)) return ROLESUB_EINVAL;
+    rs::CompressArgs a{};
+    a.shape = shape;
+    a.plan = pv;
+    a.ws = carve(w, workspace);
+    a.h = h;
+    a.v = v;
+    a.R = R_dense;
+    a.W_re = W_re;
+    a.W1 = W1;
+    a.W2 = W2;
+    a.b_re = b_re;
+    a.b1 = b1;
+    a.b2 = b2;
+    a.alpha_role = alpha_role;
+    a.alpha_lang = alpha_lang;
+    a.packed = packed_v;
+    a.idx = idx;
+    a.stream = (cudaStream_t)stream;
+    const int L = shape->num_layers, d = shape->num_heads * shape->head_dim;
+    const int64_t rows = P.rows_per_layer;
+    void *Z = static_cast<char *>(workspace) + w.total;
+    cudaError_t e = rs::launch_router(a);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    // indices 0..S-1 of k = S rows (the records it also writes are not used)
+    e = rs::launch_row_store(pv, L, idx, P.idx_bytes_per_layer, true, reinterpret_cast<uint4 *>(a.ws.row_store),
+                             a.ws.status, a.stream);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    // Z = V R (z = R^T v for every row, all d dims)
+    e = rs::launch_gemm_tc(true, L, (int)rows, d, d, v, rows * d, R_dense, (int64_t)d * d, Z, rows * d, a.ws.status,
+                           a.stream);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    return from_cuda(rs::launch_pack_dense(a, Z));
+}
+
+rolesub_status rolesub_attend_dense(const rolesub_shape *shape, const void *plan_host, const void *plan_dev,
+                                    const void *q, int64_t q_ls, int64_t q_rs, int64_t q_hs, const void *K,
+                                    int64_t k_ls, int64_t k_rs, int64_t k_hs, const void *packed_v,
+                                    const uint8_t *idx, const void *R_dense, float softmax_scale, void *o,
+                                    void *workspace, size_t ws_bytes, void *stream)
+{
+    if (!shape_ok(shape)) return ROLESUB_EINVAL;
+    PlanView pv;
+    rolesub_status st = view_plan(shape, plan_host, plan_dev, &pv);
+    if (st != ROLESUB_OK) return st;
+    if (!plan_dev) return ROLESUB_EINVAL;
+    const rolesub_plan &P = *pv.hdr;
+    const void *ptrs[] = {q, K, R_dense, o, workspace};
+    for (const void *p : ptrs)
+        if (!p || !aligned16(p)) return ROLESUB_EINVAL;
+    if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
+    if (P.idx_bytes_per_layer > 0 && !idx) return ROLESUB_EINVAL;
+    const int64_t strides[] = {q_ls, q_rs, q_hs, k_ls, k_rs, k_hs};
+    for (int64_t x : strides)
+        if (x < 0 || x % 8 != 0) return ROLESUB_EINVAL;
+    if (!isfinite(softmax_scale) || softmax_scale < 0.f) return ROLESUB_EINVAL;
+    if (!dense_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    const WsSizes w = ws_sizes(shape, pv.hdr);
+    if (ws_bytes < w.total + dense_extra_bytes(shape, pv.hdr)) return ROLESUB_EINVAL;
+    const int L = shape->num_layers, d = shape->num_heads * shape->head_dim;
+    const int64_t rows = P.rows_per_layer;
+    const size_t vals = align_up(2 * (size_t)L * (size_t)rows * d, kAlign);
+    char *Zm = static_cast<char *>(workspace) + w.total, *Vt = Zm + vals, *Rid = Vt + vals;
+    rs::AttendArgs a;
+    a.shape = shape;
+    a.plan = pv;
+    a.ws = carve(w, workspace);
+    a.q = q;
+    a.K = K;
+    a.packed = packed_v;
+    a.idx = idx;
+    a.q_ls = q_ls;
+    a.q_rs = q_rs;
+    a.q_hs = q_hs;
+    a.k_ls = k_ls;
+    a.k_rs = k_rs;
+    a.k_hs = k_hs;
+    a.scale = softmax_scale;
+    a.o = o;
+    a.stream = (cudaStream_t)stream;
+    // M z of every row, then v~ = (M z) R^T = R M z back in the original space
+    cudaError_t e = rs::launch_unpack_dense(a, Zm);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    e = rs::launch_gemm_tc(false, L, (int)rows, d, d, Zm, rows * d, R_dense, (int64_t)d * d, Vt, rows * d,
+                           a.ws.status, a.stream);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    e = rs::launch_dense_attend_prep(a, Rid);
+    if (e != cudaSuccess) return ROLESUB_ECUDA;
+    // attention over v~ as plain per-head values (every group kept, R_h = I)
+    a.packed = Vt;
+    a.packed_per_layer = rows * d;
+    a.R = Rid;
+    a.records_ready = true;
+    return from_cuda(rs::launch_attend_tc(a));
 }
 
 rolesub_status rolesub_get_device_status(const void *workspace, void *stream, int32_t *code_out,

@@ -728,7 +728,8 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
         sms = 152;
     // per-row records (kept groups, packed offset) from the caller's indices
     uint4 *recs = reinterpret_cast<uint4 *>(a.ws.row_store);
-    err = a.k_tok ? launch_row_store_budget(a.plan, L, a.idx, P.idx_bytes_per_layer, a.k_tok, recs, a.ws.status,
+    if (!a.records_ready)
+        err = a.k_tok ? launch_row_store_budget(a.plan, L, a.idx, P.idx_bytes_per_layer, a.k_tok, recs, a.ws.status,
                                             a.stream)
                   : launch_row_store(a.plan, L, const_cast<uint8_t *>(a.idx), P.idx_bytes_per_layer, false, recs,
                                      a.ws.status, a.stream);
@@ -743,7 +744,8 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
         const int64_t u1 = std::min(U, u0 + per_launch);
         const int grid = (int)std::min<int64_t>(u1 - u0, sms);
         k_attend_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(
-            tq, tk, tr, (const bf16 *)a.packed, P.packed_elems_per_layer, recs, rows, a.plan.eps_dev, E, H, qtiles,
+            tq, tk, tr, (const bf16 *)a.packed, a.packed_per_layer ? a.packed_per_layer : P.packed_elems_per_layer,
+            recs, rows, a.plan.eps_dev, E, H, qtiles,
             u0, u1, P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o, a.ws.status);
         count_launches(1);
         err = cudaGetLastError();

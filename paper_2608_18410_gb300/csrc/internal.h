@@ -71,6 +71,8 @@ struct AttendArgs {
     void *o;
     cudaStream_t stream;
     const uint8_t *k_tok = nullptr;   // per-token kept counts (budget cache), or fixed k
+    bool records_ready = false;       // ws.row_store already holds the store records
+    int64_t packed_per_layer = 0;     // values per layer of `packed`; 0: the plan's
 };
 
 // Router: language pool + per-episode bias, router GEMM, epilogue/top-k.
@@ -113,6 +115,17 @@ cudaError_t launch_row_store_budget(const PlanView &pv, int L, const uint8_t *id
 // index) in order, their indices and rows (row_bytes each).
 cudaError_t launch_select_tokens(int64_t groups, int n, int k, const float *scores, const void *x, int64_t row_bytes,
                                  int32_t *keep_idx, void *x_keep, cudaStream_t stream);
+
+// Dense rotation (one d x d R per layer): C = A B^T or A B on the tensor core
+// (gemm_tc.cu); packing of the kept d/S-wide groups of Z, the scatter of
+// M z back to [rows][d], and the attention records / identity rotations that
+// let the attention kernel read v~ = R M z as plain values (dense.cu).
+cudaError_t launch_gemm_tc(bool b_mn_major, int L, int M, int N, int K, const void *A, int64_t a_layer_stride,
+                           const void *B, int64_t b_layer_stride, void *C, int64_t c_layer_stride, int32_t *status,
+                           cudaStream_t stream);
+cudaError_t launch_pack_dense(const CompressArgs &a, const void *Z);
+cudaError_t launch_unpack_dense(const AttendArgs &a, void *Zm);
+cudaError_t launch_dense_attend_prep(const AttendArgs &a, void *R_identity);
 
 // Adds n to the process-wide launch counter (rolesub_launch_count).
 void count_launches(int n);

@@ -32,7 +32,8 @@ EXPORTS = ("rolesub_plan_size", "rolesub_layout_plan", "rolesub_workspace_size",
            "rolesub_reset_device_status", "rolesub_status_string", "rolesub_version",
            "rolesub_launch_count", "rolesub_compress_static", "rolesub_compress_additive",
            "rolesub_budget_workspace_size", "rolesub_compress_budget", "rolesub_attend_budget",
-           "rolesub_select_count", "rolesub_select_tokens")
+           "rolesub_select_count", "rolesub_select_tokens", "rolesub_dense_workspace_size",
+           "rolesub_compress_dense", "rolesub_attend_dense")
 
 STATIC_SCRATCH_BYTES = 8 << 20
 
@@ -122,6 +123,12 @@ def lib():
         L.rolesub_select_count.restype = ctypes.c_int32
         L.rolesub_select_tokens.argtypes = ([ctypes.c_int32] * 3 + [ctypes.c_double, _vp, _vp, ctypes.c_int32,
                                                                    ctypes.c_int32, _vp, _vp, _vp])
+        L.rolesub_dense_workspace_size.argtypes = [sp, _vp, _szp]
+        L.rolesub_compress_dense.argtypes = ([sp, _vp, _vp] + [_vp] * 9 + [ctypes.c_float, ctypes.c_float]
+                                             + [_vp, _vp, _vp, ctypes.c_size_t, _vp])
+        L.rolesub_attend_dense.argtypes = ([sp, _vp, _vp, _vp] + [ctypes.c_int64] * 3 + [_vp]
+                                           + [ctypes.c_int64] * 3 + [_vp, _vp, _vp, ctypes.c_float, _vp,
+                                                                     _vp, ctypes.c_size_t, _vp])
         L.rolesub_launch_count.argtypes = []
         L.rolesub_launch_count.restype = ctypes.c_uint64
         for name in EXPORTS:
@@ -202,6 +209,12 @@ class Plan:
     def budget_workspace_size(self):
         sz = ctypes.c_size_t(0)
         _check("rolesub_budget_workspace_size", lib().rolesub_budget_workspace_size(
+            ctypes.byref(self.shape), self.host_ptr, ctypes.byref(sz)))
+        return int(sz.value)
+
+    def dense_workspace_size(self):
+        sz = ctypes.c_size_t(0)
+        _check("rolesub_dense_workspace_size", lib().rolesub_dense_workspace_size(
             ctypes.byref(self.shape), self.host_ptr, ctypes.byref(sz)))
         return int(sz.value)
 
@@ -294,6 +307,24 @@ def rolesub_select_tokens(scores, x, ratio, keep_idx=None, x_keep=None, stream=N
     _check("rolesub_select_tokens", lib().rolesub_select_tokens(
         E, V, n, float(ratio), _ptr(scores), _ptr(x), hidden, dt, _ptr(keep_idx), _ptr(x_keep), _stream(stream)))
     return keep_idx[:, :, :k], x_keep[:, :, :k]
+
+
+def rolesub_compress_dense(shape, plan: Plan, plan_dev, h, v, R_dense, W_re, b_re, W1, b1, W2, b2, alpha_role,
+                           alpha_lang, packed_v, idx, workspace, ws_bytes=None, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size() if ws_bytes is None else ws_bytes
+    _check("rolesub_compress_dense", lib().rolesub_compress_dense(
+        ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(h), _ptr(v), _ptr(R_dense), _ptr(W_re),
+        _ptr(b_re), _ptr(W1), _ptr(b1), _ptr(W2), _ptr(b2), float(alpha_role), float(alpha_lang),
+        _ptr(packed_v), _ptr(idx), _ptr(workspace), int(ws_bytes), _stream(stream)))
+
+
+def rolesub_attend_dense(shape, plan: Plan, plan_dev, q, q_strides, K, k_strides, packed_v, idx, R_dense,
+                         softmax_scale, o, workspace, ws_bytes=None, stream=None):
+    ws_bytes = workspace.numel() * workspace.element_size() if ws_bytes is None else ws_bytes
+    _check("rolesub_attend_dense", lib().rolesub_attend_dense(
+        ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(q), *[int(s) for s in q_strides],
+        _ptr(K), *[int(s) for s in k_strides], _ptr(packed_v), _ptr(idx), _ptr(R_dense),
+        float(softmax_scale), _ptr(o), _ptr(workspace), int(ws_bytes), _stream(stream)))
 
 
 def rolesub_get_device_status(workspace, stream=None):
@@ -395,6 +426,39 @@ class RoleSub:
         rolesub_attend_budget(s, self.plan, self.plan_dev, q, q_strides, K, k_strides, packed, idx, k_tok, R,
                               softmax_scale, o, self.workspace, self.ws_bytes, stream)
         return o
+
+    def _dense_workspace(self):
+        if getattr(self, "_dws", None) is None:
+            n = self.plan.dense_workspace_size()
+            self._dws = self.torch.zeros(n, dtype=self.torch.uint8, device=self.device)
+        return self._dws
+
+    def compress_dense(self, h, v, R_dense, W_re, b_re, W1, b1, W2, b2, alpha_role=0.1, alpha_lang=0.1,
+                       packed=None, idx=None, stream=None):
+        """Dense-rotation compress; the first call allocates its larger
+        workspace (two [L][rows][d] bf16 buffers)."""
+        if packed is None or idx is None:
+            packed, idx = self.new_outputs()
+        ws = self._dense_workspace()
+        rolesub_compress_dense(self.shape, self.plan, self.plan_dev, h, v, R_dense, W_re, b_re, W1, b1, W2, b2,
+                               alpha_role, alpha_lang, packed, idx, ws, ws.numel(), stream)
+        return packed, idx
+
+    def attend_dense(self, q, K, packed, idx, R_dense, softmax_scale=0.0, o=None, stream=None):
+        t = self.torch
+        s = self.shape
+        d = s.num_heads * s.head_dim
+        hdr = self.plan.hdr
+        if o is None:
+            o = t.empty((s.num_layers, max(hdr.q_rows_per_layer, 1), d), dtype=self.tdtype, device=self.device)
+        ws = self._dense_workspace()
+        rolesub_attend_dense(s, self.plan, self.plan_dev, q, (hdr.q_rows_per_layer * d, d, s.head_dim), K,
+                             (hdr.rows_per_layer * d, d, s.head_dim), packed, idx, R_dense, softmax_scale, o, ws,
+                             ws.numel(), stream)
+        return o
+
+    def dense_device_status(self, stream=None):
+        return rolesub_get_device_status(self._dense_workspace(), stream)
 
     def attend(self, q, K, packed, idx, R, softmax_scale=0.0, o=None, q_strides=None, k_strides=None,
                stream=None):

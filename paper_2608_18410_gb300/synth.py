@@ -15,6 +15,9 @@ Recipe (one numpy PCG64 stream per tensor block):
   additive router (gen_additive_weights):
     W_v, W_l ~ N(0, 0.02), W_role ~ N(0, 1), b_v, b_l ~ N(0, 0.02) (fp32)
   per-token budgets (gen_priority): u ~ N(0, 1) (fp32), one C-vector per layer
+  dense rotation (gen_dense_rotation): one d x d orthonormal R per layer, Haar
+    from the QR of an fp64 Gaussian for d <= 1024, else kron(Q1, Q2) of two
+    Haar factors (64 x 64 each at d = 4096): dense and orthonormal
   R_h: Haar-random orthogonal d_h x d_h, from the QR factorisation of an
        fp64 N(0, 1) matrix with column signs fixed by sign(diag(R_qr)).
 bf16 tensors are rounded float32 -> bf16 with round-to-nearest-even and are
@@ -35,7 +38,7 @@ KINDS = ("vis", "lang", "prop", "act")
 TID = {"h": 1, "v": 2, "q": 3, "K": 4, "R": 5, "W_re": 6, "b_re": 7,
        "W1": 8, "b1": 9, "W2": 10, "b2": 11, "episodes": 12, "near_tie": 13,
        "packed": 14, "idx": 15, "W_v": 16, "b_v": 17, "W_role": 18, "W_l": 19, "b_l": 20,
-       "u": 21}
+       "u": 21, "R_dense": 22}
 
 
 @dataclasses.dataclass(frozen=True)
@@ -365,6 +368,21 @@ def gen_additive_weights(wl: Workload):
 def gen_priority(wl: Workload):
     """Priority vectors u [L][C] float32 of the per-token budget allocator."""
     return np.stack([_normal(wl.seed, layer, 0, TID["u"], (wl.C,)) for layer in range(wl.L)]).astype(np.float32)
+
+
+def gen_dense_rotation(wl: Workload):
+    """One d x d orthonormal R per layer (storage dtype), [L][d][d]."""
+    d = wl.d
+    out = np.empty((wl.L, d, d), storage_dtype(wl.dtype))
+    for layer in range(wl.L):
+        rng = _rng(wl.seed, layer, 0, TID["R_dense"])
+        if d <= 1024:
+            R = haar_orthogonal(rng, d)
+        else:
+            a = 1 << (int(np.log2(d)) // 2)
+            R = np.kron(haar_orthogonal(rng, a), haar_orthogonal(rng, d // a))
+        out[layer] = _store(R.astype(np.float32), wl.dtype)
+    return out
 
 
 def gen_packed(wl: Workload, packed_elems_per_layer: int, idx_bytes_per_layer: int, seg_table):

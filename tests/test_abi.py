@@ -241,3 +241,30 @@ def test_select_tokens_rejects_bad_arguments_before_any_launch(rsm):
     assert L.rolesub_select_tokens(1, 2, 8, 0.5, fake + 4, fake, 8, 0, fake, fake, None) == 1   # unaligned
     assert L.rolesub_select_tokens(1, 2, 20000, 0.5, fake, fake, 8, 0, fake, fake, None) == 1   # n_view too big
     assert L.rolesub_select_tokens(0, 2, 8, 0.5, None, None, 8, 0, None, None, None) == 0       # nothing to do
+
+
+def test_dense_calls_reject_bad_arguments_before_any_launch(rsm):
+    shape = rsm.make_shape(1, 4, 128, 16, 8, 32, "bf16")
+    plan = rsm.Plan(shape, [[3, 2, 0, 0]], [[4, 16, 16, 16]], [1])
+    L = rsm.lib()
+    fake = 1 << 20
+    big = plan.dense_workspace_size()
+    assert big > plan.workspace_size()
+    # shape, plan, plan_dev, h v R_dense W_re b_re W1 b1 W2 b2, alphas, packed idx ws, ws_bytes, stream
+    args = [ctypes.byref(shape), plan.host_ptr, fake] + [fake] * 9 + [0.1, 0.1, fake, fake, fake, big, None]
+    for pos in range(3, 12):
+        a = list(args)
+        a[pos] = None
+        assert L.rolesub_compress_dense(*a) == 1, pos
+    a = list(args)
+    a[17] = big - 256                   # workspace without the dense buffers
+    assert L.rolesub_compress_dense(*a) == 1
+    odd = rsm.make_shape(1, 3, 128, 16, 8, 32, "bf16")     # d = 384: not a multiple of 256
+    po = rsm.Plan(odd, [[3, 2, 0, 0]], [[4, 16, 16, 16]], [1])
+    a = list(args)
+    a[0], a[1] = ctypes.byref(odd), po.host_ptr
+    assert L.rolesub_compress_dense(*a) == 2
+    at = [ctypes.byref(shape), plan.host_ptr, fake, fake, 0, 512, 128, fake, 0, 512, 128, fake, fake, fake,
+          0.0, fake, fake, big, None]
+    at[13] = None                       # R_dense
+    assert L.rolesub_attend_dense(*at) == 1
