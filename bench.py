@@ -560,6 +560,30 @@ def run_ours(args):
     sel_bytes = 64 * 2 * (256 * 4 + sel_k * 4 + 2 * sel_k * wl.d * sel_out.element_size())
     del sel_x
 
+    # ---- the dense-rotation geometry (one d x d R per layer): compress_dense
+    # + attend_dense on the same cache, timed on their own ------------------
+    R_dense = to_dev(synth.gen_dense_rotation(wl))
+    rs.compress_dense(d["h"], d["v"], R_dense, d["W_re"], d["b_re"], d["W1"], d["b1"], d["W2"], d["b2"],
+                      wl.alpha_role, wl.alpha_lang, packed=packed, idx=idx)
+    rs.attend_dense(d["q"], d["K"], packed, idx, R_dense, o=o)
+    torch.cuda.synchronize()
+    ev_den = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+               torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    for i in range(args.steps):
+        ev_den[i][0].record(stream)
+        rs.compress_dense(d["h"], d["v"], R_dense, d["W_re"], d["b_re"], d["W1"], d["b1"], d["W2"], d["b2"],
+                          wl.alpha_role, wl.alpha_lang, packed=packed, idx=idx)
+        ev_den[i][1].record(stream)
+        rs.attend_dense(d["q"], d["K"], packed, idx, R_dense, o=o)
+        ev_den[i][2].record(stream)
+    torch.cuda.synchronize()
+    code, _ = rs.dense_device_status()
+    assert code == 0, f"device status {code}"
+    den_c_ms = statistics.mean(a.elapsed_time(b) for a, b, c in ev_den)
+    den_a_ms = statistics.mean(b.elapsed_time(c) for a, b, c in ev_den)
+    del R_dense
+    rs._dws = None
+
     # ---- one OpenVLA-OFT layer (c1), a launch-latency-bound step: eager
     # calls and the same step replayed from a CUDA graph, L2 flushed --------
     wl1 = synth.c1()
@@ -656,6 +680,13 @@ def run_ours(args):
     cab = compress_additive_bytes(wl, C_ADD)
     comp_add = {"ms": add_ms, "role_dim": C_ADD, "algorithmic_bytes": cab, "GB/s": cab / (add_ms / 1e3) / 1e9,
                 "frac": cab / (add_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
+    gemm_flop = 2.0 * wl.rows * wl.d * wl.d * wl.L     # one d x d rotation of every cache row, all layers
+    dense = {"compress_ms": den_c_ms, "attend_ms": den_a_ms,
+             "rotation_gemm_tflop": gemm_flop / 1e12,
+             "compress_tflops_rotation_only": gemm_flop / (den_c_ms / 1e3) / 1e12,
+             "attend_tflops_rotation_only": gemm_flop / (den_a_ms / 1e3) / 1e12,
+             "query_tokens_per_s_per_layer": qtok / ((den_c_ms + den_a_ms) / 1e3),
+             "r": "one d x d orthonormal R per layer (kron of two 64 x 64 Haar factors)"}
     latency = {"workload": wl1.name, "l2": "flushed before each step", "eager_ms": lat_eager,
                "graph_ms": lat_graph, "query_tokens_per_s_per_layer_graph": wl1.q_rows / (lat_graph / 1e3)}
     select = {"episodes": 64, "views": 2, "tokens_per_view": 256, "kept_per_view": sel_k, "ms": sel_ms,
@@ -676,7 +707,7 @@ def run_ours(args):
                     "ms_per_step": e2e_ms},
             "gpu_launches": launches,
             "roofline": roof, "compress": comp, "compress_additive": comp_add, "budget": budget,
-            "select_tokens": select, "latency_one_layer": latency,
+            "select_tokens": select, "latency_one_layer": latency, "dense_rotation": dense,
             "clocks": {"sm_mhz": clocks["sm_mhz"], "sm_max_mhz": clocks["sm_max_mhz"],
                        "reasons": clocks["reasons"], "samples": clocks["samples"]}}
     if ws == 1 and rank == 0 and not args.no_cpu_baseline:
