@@ -30,46 +30,55 @@ __global__ void k_lang_pool(const T *__restrict__ h, const rolesub_episode *__re
     ctx[((size_t)l * E + e) * d + col] = ep.n_lang > 0 ? s / (float)ep.n_lang : 0.f;
 }
 
-// bf16, d % 8 == 0: a thread sums eight adjacent columns (one 16-byte load
-// per row) with four rows in flight; the row order of the sum is the same
-// as above, so the result is too.
-__global__ void k_lang_pool_v8(const __nv_bfloat16 *__restrict__ h, const rolesub_episode *__restrict__ eps, int E,
-                               int64_t rows, int d, float *__restrict__ ctx)
+// bf16, d % 8 == 0: a block covers 512 columns of one (layer, episode); a
+// thread sums eight adjacent columns (one 16-byte load per row) over every
+// fourth language row, four rows in flight, and the four row classes are
+// added in a fixed order (0, 1, 2, 3) through shared memory, so the result
+// does not depend on timing.
+constexpr int kPoolParts = 4;
+
+__global__ void __launch_bounds__(256)
+k_lang_pool_v8(const __nv_bfloat16 *__restrict__ h, const rolesub_episode *__restrict__ eps, int E, int64_t rows,
+               int d, float *__restrict__ ctx)
 {
+    __shared__ float part[kPoolParts - 1][64][9];
     const int l = blockIdx.z, e = blockIdx.y;
-    const int c8 = blockIdx.x * blockDim.x + threadIdx.x;
-    if (8 * c8 >= d) return;
+    const int cl = threadIdx.x & 63, p = threadIdx.x >> 6;
+    const int c8 = blockIdx.x * 64 + cl;
+    const bool live = 8 * c8 < d;
     const rolesub_episode ep = eps[e];
     const uint4 *base = reinterpret_cast<const uint4 *>(h + ((size_t)l * rows + ep.lang_row_begin) * d) + c8;
     const size_t stride = (size_t)d / 8;
     float s[8] = {};
-    const int n = ep.n_lang;
-    int j = 0;
-    for (; j + 4 <= n; j += 4) {
-        uint4 v[4];
-#pragma unroll
-        for (int q = 0; q < 4; ++q) v[q] = __ldg(base + (size_t)(j + q) * stride);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const __nv_bfloat162 *p = reinterpret_cast<const __nv_bfloat162 *>(&v[q]);
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const float2 f = __bfloat1622float2(p[i]);
-                s[2 * i] += f.x;
-                s[2 * i + 1] += f.y;
-            }
-        }
-    }
-    for (; j < n; ++j) {
-        const uint4 v = __ldg(base + (size_t)j * stride);
-        const __nv_bfloat162 *p = reinterpret_cast<const __nv_bfloat162 *>(&v);
+    const int n = live ? ep.n_lang : 0;
+    auto add = [&](const uint4 &v) {
+        const __nv_bfloat162 *q2 = reinterpret_cast<const __nv_bfloat162 *>(&v);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
-            const float2 f = __bfloat1622float2(p[i]);
+            const float2 f = __bfloat1622float2(q2[i]);
             s[2 * i] += f.x;
             s[2 * i + 1] += f.y;
         }
+    };
+    int j = p;
+    for (; j + 3 * kPoolParts < n; j += 4 * kPoolParts) {
+        uint4 v[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) v[q] = __ldg(base + (size_t)(j + kPoolParts * q) * stride);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) add(v[q]);
     }
+    for (; j < n; j += kPoolParts) add(__ldg(base + (size_t)j * stride));
+    if (p > 0) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) part[p - 1][cl][i] = s[i];
+    }
+    __syncthreads();
+    if (p > 0 || !live) return;
+#pragma unroll
+    for (int q = 0; q < kPoolParts - 1; ++q)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) s[i] += part[q][cl][i];
     const float fn = (float)n;
 #pragma unroll
     for (int i = 0; i < 8; ++i) s[i] = n > 0 ? s[i] / fn : 0.f;
@@ -193,13 +202,69 @@ k_lang_bias(const T *__restrict__ W1, const float *__restrict__ b1, const float 
     }
 }
 
+// bf16 weights, at most kGemvEpisodes episodes (a single control step): the
+// product is a matrix-vector one, bound by reading W1_c once. A warp per
+// output f walks W1_c's row with 16-byte loads (eight weights per lane and
+// step), multiplies by the episodes' ctx in fp32 and sums the lanes with a
+// butterfly. Needs d % 8 == 0 and C % 8 == 0 (16-byte weight rows).
+constexpr int kGemvEpisodes = 4;
+
+__global__ void __launch_bounds__(256)
+k_lang_bias_gemv(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *__restrict__ ctx,
+                 int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
+{
+    const int l = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int f = blockIdx.x * 8 + warp;
+    if (f >= F) return;
+    const uint4 *w = reinterpret_cast<const uint4 *>(W1 + ((size_t)l * F + f) * (size_t)(2 * d + C) + d + C);
+    const float4 *c4 = reinterpret_cast<const float4 *>(ctx + (size_t)l * E * d);
+    const int n8 = d / 8;
+    float acc[kGemvEpisodes] = {};
+#pragma unroll 4
+    for (int k8 = lane; k8 < n8; k8 += 32) {
+        const uint4 wv = __ldg(w + k8);
+        const __nv_bfloat162 *wp = reinterpret_cast<const __nv_bfloat162 *>(&wv);
+        float wf[8];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 t = __bfloat1622float2(wp[i]);
+            wf[2 * i] = t.x;
+            wf[2 * i + 1] = t.y;
+        }
+#pragma unroll
+        for (int e = 0; e < kGemvEpisodes; ++e) {
+            if (e >= E) break;
+            const float4 x0 = __ldg(c4 + (size_t)e * (d / 4) + 2 * k8), x1 = __ldg(c4 + (size_t)e * (d / 4) + 2 * k8 + 1);
+            float a = acc[e];
+            a = fmaf(wf[0], x0.x, a);
+            a = fmaf(wf[1], x0.y, a);
+            a = fmaf(wf[2], x0.z, a);
+            a = fmaf(wf[3], x0.w, a);
+            a = fmaf(wf[4], x1.x, a);
+            a = fmaf(wf[5], x1.y, a);
+            a = fmaf(wf[6], x1.z, a);
+            a = fmaf(wf[7], x1.w, a);
+            acc[e] = a;
+        }
+    }
+#pragma unroll
+    for (int e = 0; e < kGemvEpisodes; ++e) {
+        if (e >= E) break;
+        const float v = warp_sum(acc[e]);
+        if (lane == 0) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * v;
+    }
+}
+
 // bf16 weights: the same product on the tensor cores (mma.sync m16n8k16,
 // fp32 accumulation). ctx is split into bf16 parts hi + lo (together exact to
 // about 2^-16 relative) and both are multiplied by the bf16 weights. Block:
-// 64 episodes x 64 outputs x half of d, four warps of 16 episodes each; a
-// cluster of two blocks along d adds rank 1 into rank 0 through distributed
-// shared memory. Needs d % 128 == 0 and C % 8 == 0 (16-byte weight rows).
-constexpr int kMmaSplit = 2;
+// 64 episodes x 64 outputs x 1/kSplit of d, four warps of 16 episodes each;
+// a cluster of kSplit blocks along d reduces through distributed shared
+// memory: rank r owns 8/kSplit of the eight 8-output column tiles, receives
+// every rank's partial sums for them and adds them in rank order, so the
+// result does not depend on timing. kSplit = 8 (d % 512 == 0) keeps each
+// block's walk over d short; kSplit = 2 needs d % 128 == 0. C % 8 == 0
+// (16-byte weight rows) in both.
 
 __device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2, uint32_t &r3)
 {
@@ -223,7 +288,8 @@ __device__ __forceinline__ uint32_t pack2(float a, float b)
     return *reinterpret_cast<const uint32_t *>(&v);
 }
 
-__global__ void __cluster_dims__(kMmaSplit, 1, 1) __launch_bounds__(128)
+template <int kSplit>
+__global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(128)
 k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *__restrict__ ctx,
                 int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
 {
@@ -235,8 +301,8 @@ k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ 
     const uint32_t sA1 = sA0 + BE * BK * 2, sBs = sA1 + BE * BK * 2;
     const int l = blockIdx.z, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t rank = cluster_rank();
-    const int f0 = (blockIdx.x / kMmaSplit) * BF, e0 = blockIdx.y * BE;
-    const int kper = d / kMmaSplit;
+    const int f0 = (blockIdx.x / kSplit) * BF, e0 = blockIdx.y * BE;
+    const int kper = d / kSplit;
     const int kb = (int)rank * kper, ke = kb + kper;
     const size_t wstride = (size_t)(2 * d + C);
     const __nv_bfloat16 *wbase = W1 + (size_t)l * F * wstride + d + C;
@@ -305,33 +371,50 @@ k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ 
             }
         }
     }
-    // rank 1 adds its sums into rank 0 (thread-major, 128 x 32 floats)
+    // every rank sends column tiles j of its sums to the rank that owns them:
+    // slot ((q * 128 + tid) * J + jj) of rank r holds rank q's tile r J + jj
+    constexpr int J = 8 / kSplit;
+    static_assert(kSplit * 128 * J * 16 <= (int)sizeof(sm), "reduction buffer");
     __syncthreads();
     cluster_sync();
-    if (rank != 0) {
-        const uint32_t local = sA0 + 4u * ((uint32_t)tid * 32u);
-        uint32_t remote;
-        asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"(0u));
+    {
+        const uint32_t local = sA0 + 16u * ((rank * 128u + (uint32_t)tid) * (uint32_t)J);
 #pragma unroll
-        for (int q = 0; q < 32; ++q)
-            asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(remote + 4u * q), "f"(acc[q >> 2][q & 3]) : "memory");
+        for (int r = 0; r < kSplit; ++r) {
+            uint32_t remote;
+            asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(local), "r"((uint32_t)r));
+#pragma unroll
+            for (int jj = 0; jj < J; ++jj)
+                asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote + 16u * jj),
+                             "f"(acc[r * J + jj][0]), "f"(acc[r * J + jj][1]), "f"(acc[r * J + jj][2]),
+                             "f"(acc[r * J + jj][3])
+                             : "memory");
+        }
     }
     cluster_sync();
-    if (rank != 0) return;
-    const float *red = reinterpret_cast<const float *>(sm) + tid * 32;
-#pragma unroll
-    for (int q = 0; q < 32; ++q) acc[q >> 2][q & 3] += red[q];
+    const float4 *red = reinterpret_cast<const float4 *>(sm);
     const int g = lane >> 2, t2 = 2 * (lane & 3);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int jj = 0; jj < J; ++jj) {
+        float4 v = red[tid * J + jj];
 #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-            const int e = e0 + 16 * warp + g + 8 * h;
+        for (int q = 1; q < kSplit; ++q) {
+            const float4 w = red[(q * 128 + tid) * J + jj];
+            v.x += w.x;
+            v.y += w.y;
+            v.z += w.z;
+            v.w += w.w;
+        }
+        const float o[4] = {v.x, v.y, v.z, v.w};
+        const int j = (int)rank * J + jj;
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+            const int e = e0 + 16 * warp + g + 8 * hh;
             if (e >= E) continue;
 #pragma unroll
             for (int q = 0; q < 2; ++q) {
                 const int f = f0 + 8 * j + t2 + q;
-                if (f < F) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * acc[j][2 * h + q];
+                if (f < F) beta[((size_t)l * E + e) * F + f] = b1[(size_t)l * F + f] + alpha_lang * o[2 * hh + q];
             }
         }
     }
@@ -480,7 +563,7 @@ cudaError_t launch_lang_pool(const CompressArgs &a)
     const rolesub_plan &P = *a.plan.hdr;
     const int L = S.num_layers, E = P.num_episodes, d = S.num_heads * S.head_dim;
     if (S.dtype == ROLESUB_BF16 && d % 8 == 0 && ((uintptr_t)a.h & 15) == 0)
-        k_lang_pool_v8<<<dim3((d / 8 + 127) / 128, E, L), 128, 0, a.stream>>>(
+        k_lang_pool_v8<<<dim3((d / 8 + 63) / 64, E, L), 256, 0, a.stream>>>(
             (const __nv_bfloat16 *)a.h, a.plan.eps_dev, E, P.rows_per_layer, d, a.ws.lang_ctx);
     else if (S.dtype == ROLESUB_BF16)
         k_lang_pool<__nv_bfloat16><<<dim3((d + 255) / 256, E, L), 256, 0, a.stream>>>(
@@ -505,8 +588,14 @@ static cudaError_t launch_router_t(const CompressArgs &a)
             *W2 = (const T *)a.W2;
     cudaError_t err = launch_lang_pool(a);
     if (err != cudaSuccess) return err;
-    if (sizeof(T) == 2 && d % 128 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
-        k_lang_bias_mma<<<dim3((F + 63) / 64 * kMmaSplit, (E + 63) / 64, L), 128, 0, a.stream>>>(
+    if (sizeof(T) == 2 && E <= kGemvEpisodes && d % 8 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
+        k_lang_bias_gemv<<<dim3((F + 7) / 8, L), 256, 0, a.stream>>>(
+            (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+    else if (sizeof(T) == 2 && d % 512 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
+        k_lang_bias_mma<8><<<dim3((F + 63) / 64 * 8, (E + 63) / 64, L), 128, 0, a.stream>>>(
+            (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+    else if (sizeof(T) == 2 && d % 128 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
+        k_lang_bias_mma<2><<<dim3((F + 63) / 64 * 2, (E + 63) / 64, L), 128, 0, a.stream>>>(
             (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
     else
         k_lang_bias<T><<<dim3((F + 31) / 32 * kBiasSplit, (E + 63) / 64, L), 256, 0, a.stream>>>(

@@ -1,12 +1,14 @@
 // router_tc.cu -- role-conditioned group scores and top-k on the
 // 5th-generation tensor core (Sec. 3.3-3.4), bf16 inputs.
 //
-// One CTA per (128-row router tile, layer), 192 threads:
-//   warp 4  TMA producer, warp 5  MMA issuer, warps 0-3  epilogue (a
-//   thread per tile row / TMEM lane).
+// One CTA per (128-row router tile, layer), 320 threads:
+//   warp 4  TMA producer, warp 5  MMA issuer, warps 0-3 and 6-9  epilogue:
+//   two threads per tile row / TMEM lane (warp w reads lane quadrant w % 4),
+//   each taking half of the row's role and hidden columns.
 // Mainloop over the hidden size d in 64-column blocks (4-stage TMA ring of
-// 56 KB stages; the epilogue's weights W1_a and W2 are loaded into the
-// drained ring once the last products have read it):
+// 56 KB stages; the epilogue's weights W1_a and W2 are loaded into stage 0
+// as soon as its last products have read it, three blocks before the end,
+// and the epilogue's operands go into stages 1-3 once the mainloop is done):
 //   TMEM[0,256)   += h W1_h^T      (first d input columns of W1)
 //   TMEM[256,320) += h W_re^T      (role logits)
 // Epilogue, per routed row i:
@@ -34,7 +36,7 @@ namespace {
 using namespace sm100;
 typedef __nv_bfloat16 bf16;
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;
 constexpr int kRows = 128;
 constexpr int kF = 256;      // router hidden
 constexpr int kC = 64;       // role dim
@@ -42,28 +44,31 @@ constexpr int kG = 16;       // groups
 constexpr int kStages = 4;
 
 constexpr uint32_t kStageBytes = 16384 + 32768 + 8192;       // A | W1_h | W_re
-// epilogue weights go into the drained ring after the main loop, above the
-// epilogue's own operands (which use [0, 160K))
-constexpr uint32_t kOffW1A = 163840;                         // 160K: W1_a [256][64]
-constexpr uint32_t kOffW2 = kOffW1A + 32768;                 // 192K: W2 [16][256]
 constexpr uint32_t kOffBar = kStages * kStageBytes;          // 224K
-static_assert(kOffW2 + 8192 <= kOffBar, "epilogue weights inside the ring");
 constexpr uint32_t kSmemBytes = kOffBar + 256 + 1024;
-// epilogue operands reuse the (drained) stage ring
-constexpr uint32_t kOffARhi = 0, kOffARlo = 16384, kOffUhi = 32768, kOffUlo = 98304;
+// epilogue weights in stage 0: W1_a [256][64], W2 [16][256]
+constexpr uint32_t kOffW1A = 0, kOffW2 = 32768;
+static_assert(kOffW2 + 8192 <= kStageBytes, "epilogue weights inside stage 0");
+// epilogue operands in stages 1-3 (1024-byte aligned for the 128-byte
+// swizzle): alpha_role a hi / lo [128][64], u hi / lo [128][256]
+constexpr uint32_t kOffARhi = kStageBytes, kOffARlo = kOffARhi + 16384, kOffUhi = kOffARlo + 16384,
+                   kOffUlo = kOffUhi + 65536;
+// role-softmax partial max / sum of each half row: [2][2][128] floats
+constexpr uint32_t kOffXch = kOffUlo + 65536;
+static_assert(kOffXch + 2048 <= kOffBar, "epilogue operands inside stages 1-3");
 
 constexpr uint32_t kIdescH = idesc_bf16(128, 256, false);
 constexpr uint32_t kIdescR = idesc_bf16(128, 64, false);
 constexpr uint32_t kIdescG = idesc_bf16(128, 16, false);
 
-__device__ __forceinline__ void split_bf16(float x, float &hi_out, uint16_t &hi, uint16_t &lo)
+// x0, x1 -> bf16 pairs hi = rn(x), lo = rn(x - hi) (x0 in the low halves)
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t &hi, uint32_t &lo)
 {
-    const bf16 h = __float2bfloat16_rn(x);
-    const float hf = __bfloat162float(h);
-    const bf16 l = __float2bfloat16_rn(x - hf);
-    hi = *reinterpret_cast<const uint16_t *>(&h);
-    lo = *reinterpret_cast<const uint16_t *>(&l);
-    hi_out = hf;
+    const __nv_bfloat162 h = __floats2bfloat162_rn(x0, x1);
+    hi = *reinterpret_cast<const uint32_t *>(&h);
+    const float h0 = __uint_as_float(hi << 16), h1 = __uint_as_float(hi & 0xffff0000u);
+    const __nv_bfloat162 l2 = __floats2bfloat162_rn(x0 - h0, x1 - h1);
+    lo = *reinterpret_cast<const uint32_t *>(&l2);
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -78,6 +83,7 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
     __shared__ volatile int abort_flag;
     const uint32_t sraw = smem_u32(smem_raw);
     const uint32_t sb = (sraw + 1023u) & ~1023u;
+    uint8_t *sp = smem_raw + (sb - sraw);
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int l = blockIdx.y;
     const int row0 = plan.route_tiles[blockIdx.x];
@@ -93,9 +99,9 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
         for (int i = 0; i < 2 * kStages; ++i) mbar_init(bar_full + 8 * i, 1);
         mbar_init(bar_acc, 1);
         mbar_init(bar_w, 1);
-        mbar_init(bar_ar, 128);
+        mbar_init(bar_ar, 256);
         mbar_init(bar_h, 1);
-        mbar_init(bar_u, 128);
+        mbar_init(bar_u, 256);
         mbar_init(bar_g, 1);
         fence_mbar_init();
     }
@@ -129,12 +135,11 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
                 tma_load_3d(st + 49152, &tm_wre, 64 * kb, 0, l, bar_full + 8 * s);
             }
             // epilogue weights of this layer, W1_a (input columns d..d+C) and
-            // W2, into stages 2 and 3 once their last products are done
-            for (int s = 2; s < kStages && ok; ++s)
-                if (nkb > s) {
-                    const int last = s + kStages * ((nkb - 1 - s) / kStages);
-                    ok = mbar_wait(bar_empty + 8 * s, (last / kStages) & 1, status, &abort_flag, 28);
-                }
+            // W2, into stage 0 once its last products are done
+            if (ok && nkb > 0) {
+                const int last = kStages * ((nkb - 1) / kStages);
+                ok = mbar_wait(bar_empty, (last / kStages) & 1, status, &abort_flag, 28);
+            }
             if (ok) {
                 mbar_expect_tx(bar_w, 32768 + 8192);
                 tma_load_3d(sb + kOffW1A, &tm_w1, d, 0, l, bar_w);
@@ -185,87 +190,91 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
             mma_commit(bar_g);
         }
     } else {
-        // ------------------------------------------------ epilogue warps 0-3
-        const int64_t r = (int64_t)row0 + tid;
+        // ------------------------------------------- epilogue warps 0-3, 6-9
+        const int quad = warp & 3, half = warp >= 6 ? 1 : 0;
+        const int row = 32 * quad + lane;
+        const int64_t r = (int64_t)row0 + row;
         bool routed = false;
         rolesub_segment sg{};
         if (r < rows) {
             sg = plan.segs[plan.row_seg[r]];
             routed = sg.k > 0 && sg.k < G;
         }
-        const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
-        const uint32_t swz = (uint32_t)(tid & 7);
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
+        const uint32_t swz = (uint32_t)(row & 7);
+        float *xch = reinterpret_cast<float *>(sp + kOffXch);
         mbar_wait(bar_acc, 0, status, &abort_flag, 25);
         tc_fence_after();
         __syncwarp();
-        // role softmax -> alpha_role * a, split into bf16 hi / lo operand rows
+        // role softmax over the two halves (max and sum exchanged through
+        // shared memory, the halves' sums added in order) -> alpha_role * a
+        // as bf16 hi / lo operand rows
         {
             uint32_t sr[32];
-            float lg[kC];
+            tmem_ld32(lane_base + 256 + 32 * half, sr);
+            tmem_wait_ld();
+            const float4 *bre = reinterpret_cast<const float4 *>(b_re + (int64_t)l * kC + 32 * half);
+            float lg[32];
 #pragma unroll
-            for (int q = 0; q < 2; ++q) {
-                tmem_ld32(lane_base + 256 + 32 * q, sr);
-                tmem_wait_ld();
-#pragma unroll
-                for (int j = 0; j < 32; ++j) lg[32 * q + j] = __uint_as_float(sr[j]) + __ldg(b_re + (int64_t)l * kC + 32 * q + j);
+            for (int q = 0; q < 8; ++q) {
+                const float4 bb = __ldg(bre + q);
+                lg[4 * q] = __uint_as_float(sr[4 * q]) + bb.x;
+                lg[4 * q + 1] = __uint_as_float(sr[4 * q + 1]) + bb.y;
+                lg[4 * q + 2] = __uint_as_float(sr[4 * q + 2]) + bb.z;
+                lg[4 * q + 3] = __uint_as_float(sr[4 * q + 3]) + bb.w;
             }
             float mx = -INFINITY;
 #pragma unroll
-            for (int c = 0; c < kC; ++c) mx = fmaxf(mx, lg[c]);
+            for (int c = 0; c < 32; ++c) mx = fmaxf(mx, lg[c]);
+            xch[128 * half + row] = mx;
+            named_bar(1 + quad, 64);
+            mx = fmaxf(xch[row], xch[128 + row]);
             float sum = 0.f;
 #pragma unroll
-            for (int c = 0; c < kC; ++c) {
+            for (int c = 0; c < 32; ++c) {
                 lg[c] = expf(lg[c] - mx);
                 sum += lg[c];
             }
-            const float sc = alpha_role / sum;
+            xch[256 + 128 * half + row] = sum;
+            named_bar(1 + quad, 64);
+            const float sc = alpha_role / (xch[256 + row] + xch[384 + row]);
 #pragma unroll
-            for (int cc = 0; cc < 8; ++cc) {
+            for (int cc = 0; cc < 4; ++cc) {
                 uint32_t hw[4], lw[4];
 #pragma unroll
-                for (int p = 0; p < 4; ++p) {
-                    float dummy;
-                    uint16_t h0, l0, h1, l1;
-                    split_bf16(lg[8 * cc + 2 * p] * sc, dummy, h0, l0);
-                    split_bf16(lg[8 * cc + 2 * p + 1] * sc, dummy, h1, l1);
-                    hw[p] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-                    lw[p] = (uint32_t)l0 | ((uint32_t)l1 << 16);
-                }
-                const uint32_t off = (uint32_t)tid * 128u + (((uint32_t)cc ^ swz) << 4);
+                for (int p = 0; p < 4; ++p) split_pair(lg[8 * cc + 2 * p] * sc, lg[8 * cc + 2 * p + 1] * sc, hw[p], lw[p]);
+                const uint32_t off = (uint32_t)row * 128u + (((uint32_t)(4 * half + cc) ^ swz) << 4);
                 st_shared_v4(sb + kOffARhi + off, hw[0], hw[1], hw[2], hw[3]);
                 st_shared_v4(sb + kOffARlo + off, lw[0], lw[1], lw[2], lw[3]);
             }
         }
         fence_async_smem();
         mbar_arrive(bar_ar);
-        // u = ReLU(hidden + beta_e), split into bf16 hi / lo operand rows
+        // u = ReLU(hidden + beta_e) on this half's 128 columns, split into
+        // bf16 hi / lo operand rows
         mbar_wait(bar_h, 0, status, &abort_flag, 26);
         tc_fence_after();
         __syncwarp();
         {
-            const float *be = beta + ((int64_t)l * E + sg.episode) * kF;
+            const float4 *be = reinterpret_cast<const float4 *>(beta + ((int64_t)l * E + sg.episode) * kF + 128 * half);
 #pragma unroll 1
-            for (int q = 0; q < 8; ++q) {
+            for (int q = 0; q < 4; ++q) {
                 uint32_t sr[32];
-                tmem_ld32(lane_base + 32 * q, sr);
+                tmem_ld32(lane_base + 128 * half + 32 * q, sr);
                 tmem_wait_ld();
 #pragma unroll
                 for (int cc = 0; cc < 4; ++cc) {
+                    const float4 b0 = __ldg(be + 8 * q + 2 * cc), b1 = __ldg(be + 8 * q + 2 * cc + 1);
+                    const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
                     uint32_t hw[4], lw[4];
 #pragma unroll
                     for (int p = 0; p < 4; ++p) {
                         const int j = 8 * cc + 2 * p;
-                        const float u0 = fmaxf(__uint_as_float(sr[j]) + (routed ? __ldg(be + 32 * q + j) : 0.f), 0.f);
-                        const float u1 = fmaxf(__uint_as_float(sr[j + 1]) + (routed ? __ldg(be + 32 * q + j + 1) : 0.f), 0.f);
-                        float dummy;
-                        uint16_t h0, l0, h1, l1;
-                        split_bf16(u0, dummy, h0, l0);
-                        split_bf16(u1, dummy, h1, l1);
-                        hw[p] = (uint32_t)h0 | ((uint32_t)h1 << 16);
-                        lw[p] = (uint32_t)l0 | ((uint32_t)l1 << 16);
+                        split_pair(fmaxf(__uint_as_float(sr[j]) + bb[2 * p], 0.f),
+                                   fmaxf(__uint_as_float(sr[j + 1]) + bb[2 * p + 1], 0.f), hw[p], lw[p]);
                     }
-                    const int chunk = 4 * q + cc;   // 16-byte chunk of the 256-column row
-                    const uint32_t off = (uint32_t)(chunk >> 3) * 16384u + (uint32_t)tid * 128u +
+                    const int chunk = 16 * half + 4 * q + cc;   // 16-byte chunk of the 256-column row
+                    const uint32_t off = (uint32_t)(chunk >> 3) * 16384u + (uint32_t)row * 128u +
                                          (((uint32_t)(chunk & 7) ^ swz) << 4);
                     st_shared_v4(sb + kOffUhi + off, hw[0], hw[1], hw[2], hw[3]);
                     st_shared_v4(sb + kOffUlo + off, lw[0], lw[1], lw[2], lw[3]);
@@ -274,27 +283,36 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
         }
         fence_async_smem();
         mbar_arrive(bar_u);
-        // gamma + b2 -> top-k
-        mbar_wait(bar_g, 0, status, &abort_flag, 27);
-        tc_fence_after();
-        __syncwarp();
-        uint32_t sr[32];
-        tmem_ld32(lane_base + 320, sr);
-        tmem_wait_ld();
-        if (routed && !abort_flag) {
-            float gam[kG];
+        // gamma + b2 -> top-k (first half)
+        if (half == 0) {
+            mbar_wait(bar_g, 0, status, &abort_flag, 27);
+            tc_fence_after();
+            __syncwarp();
+            uint32_t sr[32];
+            tmem_ld32(lane_base + 320, sr);
+            tmem_wait_ld();
+            if (routed && !abort_flag) {
+                const float4 *b24 = reinterpret_cast<const float4 *>(b2 + (int64_t)l * kG);
+                float gam[kG];
 #pragma unroll
-            for (int g = 0; g < kG; ++g) gam[g] = __uint_as_float(sr[g]) + __ldg(b2 + (int64_t)l * kG + g);
-            const int k = sg.k;
-            uint8_t *dst = idx + (int64_t)l * idx_per_layer + sg.idx_off + (r - sg.token_row) * k;
-            int pos = 0;
+                for (int q = 0; q < kG / 4; ++q) {
+                    const float4 bb = __ldg(b24 + q);
+                    gam[4 * q] = __uint_as_float(sr[4 * q]) + bb.x;
+                    gam[4 * q + 1] = __uint_as_float(sr[4 * q + 1]) + bb.y;
+                    gam[4 * q + 2] = __uint_as_float(sr[4 * q + 2]) + bb.z;
+                    gam[4 * q + 3] = __uint_as_float(sr[4 * q + 3]) + bb.w;
+                }
+                const int k = sg.k;
+                uint8_t *dst = idx + (int64_t)l * idx_per_layer + sg.idx_off + (r - sg.token_row) * k;
+                int pos = 0;
 #pragma unroll
-            for (int g = 0; g < kG; ++g) {
-                int rank = 0;
+                for (int g = 0; g < kG; ++g) {
+                    int rank = 0;
 #pragma unroll
-                for (int g2 = 0; g2 < kG; ++g2)
-                    rank += (gam[g2] > gam[g] || (gam[g2] == gam[g] && g2 < g)) ? 1 : 0;
-                if (rank < k && pos < k) dst[pos++] = (uint8_t)g;   // pos < k: NaN-safe
+                    for (int g2 = 0; g2 < kG; ++g2)
+                        rank += (gam[g2] > gam[g] || (gam[g2] == gam[g] && g2 < g)) ? 1 : 0;
+                    if (rank < k && pos < k) dst[pos++] = (uint8_t)g;   // pos < k: NaN-safe
+                }
             }
         }
     }
