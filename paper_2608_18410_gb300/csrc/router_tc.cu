@@ -94,7 +94,8 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
     const uint32_t bar_full = sb + kOffBar;                  // [kStages]
     const uint32_t bar_empty = bar_full + 8 * kStages;       // [kStages]
     const uint32_t bar_acc = bar_empty + 8 * kStages, bar_w = bar_acc + 8, bar_ar = bar_acc + 16,
-                   bar_h = bar_acc + 24, bar_u = bar_acc + 32, bar_g = bar_acc + 40, bar_s = bar_acc + 48;
+                   bar_h = bar_acc + 24, bar_g = bar_acc + 32, bar_s = bar_acc + 40;
+    const uint32_t bar_u = bar_acc + 48;   // [4]: u staged for K columns [32q, 32q + 32) of both halves
 
     if (tid == 0) {
         abort_flag = 0;
@@ -103,7 +104,7 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
         mbar_init(bar_w, 1);
         mbar_init(bar_ar, 256);
         mbar_init(bar_h, 1);
-        mbar_init(bar_u, 256);
+        for (int q = 0; q < 4; ++q) mbar_init(bar_u + 8 * q, 256);
         mbar_init(bar_g, 1);
         mbar_init(bar_s, 128);
         fence_mbar_init();
@@ -143,6 +144,15 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
                     tma_load_3d(st + 16384, &tm_w1, 64 * kb, 0, l, bar_full + 8 * s);
                     tma_load_3d(st + 49152, &tm_wre, 64 * kb, 0, l, bar_full + 8 * s);
                 }
+                // the next item's first token blocks into L2 while this
+                // item's last products and epilogue run
+                {
+                    const int tn = t + (int)gridDim.x;
+                    if (ok && tn < total) {
+                        const int ln = tn / tiles, rn = plan.route_tiles[tn - ln * tiles];
+                        for (int kb = 0; kb < kStages && kb < nkb; ++kb) tma_prefetch_l2_3d(&tm_h, 64 * kb, rn, ln);
+                    }
+                }
                 // epilogue weights of this layer, W1_a (input columns d..d+C)
                 // and W2, into stage 0 once its last products are done
                 if (ok && g > 0) {
@@ -163,7 +173,7 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
             for (int t = blockIdx.x, it = 0; t < total && ok; t += gridDim.x, ++it) {
                 const uint32_t ph = (uint32_t)it & 1u;
                 // TMEM [0, 320) is free again: the previous item's epilogue
-                // read it before arriving at bar_u, waited for below
+                // read it before arriving at bar_u[3], waited for below
                 for (int kb = 0; kb < nkb; ++kb, ++g) {
                     const uint32_t s = g % kStages;
                     if (!mbar_wait(bar_full + 8 * s, (g / kStages) & 1, status, &abort_flag, 21)) {
@@ -194,20 +204,29 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
                         mma_bf16(tmem, sdesc_sw128(sb + (part ? kOffARlo : kOffARhi) + 32u * kk, 16, 1024),
                                  sdesc_sw128(sb + kOffW1A + 32u * kk, 16, 1024), kIdescH, 1u);
                 mma_commit(bar_h);
-                // gamma = u W2^T, hi and lo parts, once the previous item's
-                // scores have been read
-                if (!mbar_wait(bar_u, ph, status, &abort_flag, 24)) break;
+                // gamma = u W2^T, hi and lo parts, a quarter of K at a time
+                // as the epilogue stages u, once the previous item's scores
+                // have been read
                 if (it > 0 && !mbar_wait(bar_s, ph ^ 1u, status, &abort_flag, 30)) break;
-                tc_fence_after();
-#pragma unroll
-                for (int part = 0; part < 2; ++part)
-#pragma unroll
-                    for (int kk = 0; kk < 16; ++kk) {
-                        const uint32_t ao = (part ? kOffUlo : kOffUhi) + (kk >> 2) * 16384u + (kk & 3) * 32u;
-                        const uint32_t bo = kOffW2 + (kk >> 2) * 2048u + (kk & 3) * 32u;
-                        mma_bf16(tmem + 320, sdesc_sw128(sb + ao, 16, 1024), sdesc_sw128(sb + bo, 16, 1024), kIdescG,
-                                 (part > 0 || kk > 0) ? 1u : 0u);
+                for (int q = 0; q < 4 && ok; ++q) {
+                    if (!mbar_wait(bar_u + 8 * q, ph, status, &abort_flag, 24)) {
+                        ok = false;
+                        break;
                     }
+                    tc_fence_after();
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int kk = 2 * q + (i & 1) + 8 * (i >> 1);   // K16 steps of quarter q, both halves
+#pragma unroll
+                        for (int part = 0; part < 2; ++part) {
+                            const uint32_t ao = (part ? kOffUlo : kOffUhi) + (kk >> 2) * 16384u + (kk & 3) * 32u;
+                            const uint32_t bo = kOffW2 + (kk >> 2) * 2048u + (kk & 3) * 32u;
+                            mma_bf16(tmem + 320, sdesc_sw128(sb + ao, 16, 1024), sdesc_sw128(sb + bo, 16, 1024),
+                                     kIdescG, (q > 0 || i > 0 || part > 0) ? 1u : 0u);
+                        }
+                    }
+                }
+                if (!ok) break;
                 mma_commit(bar_g);
             }
         }
@@ -230,6 +249,15 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
             if (r < rows) {
                 sg = plan.segs[plan.row_seg[r]];
                 routed = sg.k > 0 && sg.k < G;
+            }
+            // this row's bias lines into L1 while the products run: beta_e
+            // (this half's 128 columns), b_re (32), b2
+            {
+                const float *be = beta + ((int64_t)l * E + sg.episode) * kF + 128 * half;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) prefetch_l1(be + 32 * i);
+                prefetch_l1(b_re + (int64_t)l * kC + 32 * half);
+                prefetch_l1(b2 + (int64_t)l * kG);
             }
             mbar_wait(bar_acc, ph, status, &abort_flag, 25);
             tc_fence_after();
@@ -309,13 +337,14 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
                         st_shared_v4(sb + kOffUhi + off, hw[0], hw[1], hw[2], hw[3]);
                         st_shared_v4(sb + kOffUlo + off, lw[0], lw[1], lw[2], lw[3]);
                     }
+                    // quarter q staged; after the last one TMEM [0, 320)
+                    // has been read and the next item's products may
+                    // overwrite it
+                    tc_fence_before();
+                    fence_async_smem();
+                    mbar_arrive(bar_u + 8 * q);
                 }
             }
-            // TMEM [0, 320) has been read: the next item's products may
-            // overwrite it once every thread has arrived
-            tc_fence_before();
-            fence_async_smem();
-            mbar_arrive(bar_u);
             // gamma + b2 -> top-k (first half)
             if (half == 0) {
                 mbar_wait(bar_g, ph, status, &abort_flag, 27);
