@@ -426,6 +426,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
         // groups of this thread's row that may be non-zero, per Z slot (16 bits
         // each); a slot's first use clears everything
         uint64_t dirty = ~0ull;
+        pdl_wait();   // the row records come from the kernel before this one
         ChunkIt it = first;
         uint32_t g = (uint32_t)par;
         if (par) it_next(sp, it, nu);
@@ -743,12 +744,21 @@ cudaError_t launch_attend_tc(const AttendArgs &a)
     for (int64_t u0 = 0; u0 < U; u0 += per_launch) {
         const int64_t u1 = std::min(U, u0 + per_launch);
         const int grid = (int)std::min<int64_t>(u1 - u0, sms);
-        k_attend_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(
-            tq, tk, tr, (const bf16 *)a.packed, a.packed_per_layer ? a.packed_per_layer : P.packed_elems_per_layer,
-            recs, rows, a.plan.eps_dev, E, H, qtiles,
-            u0, u1, P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o, a.ws.status);
+        const int64_t ppl = a.packed_per_layer ? a.packed_per_layer : P.packed_elems_per_layer;
+        if (!a.records_ready) {
+            // a dependent of the record kernel: queries, keys and R_h are the
+            // caller's, only the gather waits for the records
+            err = launch_pdl(k_attend_tc, dim3(grid), dim3(kThreads), kSmemBytes, a.stream, tq, tk, tr,
+                             (const bf16 *)a.packed, ppl, (const uint4 *)recs, rows, a.plan.eps_dev, E, H, qtiles,
+                             u0, u1, (int64_t)P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o,
+                             a.ws.status);
+        } else {
+            k_attend_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(
+                tq, tk, tr, (const bf16 *)a.packed, ppl, recs, rows, a.plan.eps_dev, E, H, qtiles, u0, u1,
+                P.q_rows_per_layer, scale * 1.4426950408889634f, (bf16 *)a.o, a.ws.status);
+            err = cudaGetLastError();
+        }
         count_launches(1);
-        err = cudaGetLastError();
         if (err != cudaSuccess) return err;
     }
     return cudaSuccess;

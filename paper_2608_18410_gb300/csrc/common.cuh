@@ -5,12 +5,40 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "rolesub.h"
 
 namespace rs {
 
 // Status word at the start of every workspace: {code, detail}.
 constexpr size_t kStatusBytes = 256;
+
+// Programmatic dependent launch. A kernel started by launch_pdl may begin
+// while its predecessor in the stream still runs: it must call pdl_wait()
+// before touching anything the predecessor writes (pdl_wait returns once the
+// predecessor has completed and its writes are visible; at once for a kernel
+// launched the ordinary way). pdl_trigger() lets this kernel's own dependent
+// be scheduled early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+template <class... P, class... A>
+inline cudaError_t launch_pdl(void (*kern)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                              A &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<A>(args)...);
+}
 
 __device__ __forceinline__ void report(int32_t *status, int32_t code, int32_t detail)
 {

@@ -92,8 +92,10 @@ bool router_tc_supported(const rolesub_shape *s);
 cudaError_t launch_router_tc(const CompressArgs &a);
 // 16-byte per-(layer, row) store records (kept group ids, packed offset, k)
 // from the group indices; write_identity also fills indices of k = S rows.
+// pdl: launched as a programmatic dependent of the kernel before it.
 cudaError_t launch_row_store(const PlanView &pv, int L, uint8_t *idx, int64_t idx_per_layer,
-                             bool write_identity, uint4 *recs, int32_t *status, cudaStream_t stream);
+                             bool write_identity, uint4 *recs, int32_t *status, cudaStream_t stream,
+                             bool pdl = false);
 // Rotation and packing on tcgen05/TMA (bf16, d_h = 128, S = 16).
 bool rotate_tc_supported(const rolesub_shape *s);
 cudaError_t launch_rotate_tc(const CompressArgs &a);

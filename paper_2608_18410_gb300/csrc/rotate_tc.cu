@@ -55,6 +55,8 @@ __global__ void __launch_bounds__(256)
 k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_per_layer, bool write_identity,
             uint4 *__restrict__ meta, int32_t *status)
 {
+    pdl_trigger();
+    pdl_wait();   // idx may come from the kernel just before
     const int l = blockIdx.y;
     const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (r >= rows) return;
@@ -167,6 +169,9 @@ k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CU
         }
     } else {
         const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
+        // the records (and the indices behind them) come from the kernels
+        // before this one, which may still run while the first products do
+        pdl_wait();
         // row records of this thread's row in tiles t, t+1 (t+2 is fetched
         // during tile t, so the load latency hides behind two tiles of work)
         const uint4 *mrow = meta + (int64_t)l * rows + (int64_t)t0 * kRows + tid;
@@ -262,25 +267,39 @@ cudaError_t launch_rotate_tc(const CompressArgs &a)
     splits = (ntiles + per - 1) / per;
     uint4 *meta = reinterpret_cast<uint4 *>(a.ws.row_store);
     if (!a.records_ready) {
-        err = launch_row_store(a.plan, L, a.idx, P.idx_bytes_per_layer, true, meta, a.ws.status, a.stream);
+        // the records and then the products start while the router's tail
+        // still runs; both wait for their predecessor before reading its output
+        err = launch_row_store(a.plan, L, a.idx, P.idx_bytes_per_layer, true, meta, a.ws.status, a.stream, true);
         if (err != cudaSuccess) return err;
+        err = launch_pdl(k_rotate_tc, dim3(H, L, splits), dim3(kThreads), kSmemBytes, a.stream, tv, tr,
+                         (const uint4 *)meta, rows, H, per, ntiles, (bf16 *)a.packed,
+                         (int64_t)P.packed_elems_per_layer, a.ws.status);
+    } else {
+        k_rotate_tc<<<dim3(H, L, splits), kThreads, kSmemBytes, a.stream>>>(
+            tv, tr, meta, rows, H, per, ntiles, (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
+        err = cudaGetLastError();
     }
-    k_rotate_tc<<<dim3(H, L, splits), kThreads, kSmemBytes, a.stream>>>(
-        tv, tr, meta, rows, H, per, ntiles, (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
     count_launches(1);
-    return cudaGetLastError();
+    return err;
 }
 
 cudaError_t launch_row_store(const PlanView &pv, int L, uint8_t *idx, int64_t idx_per_layer, bool write_identity,
-                             uint4 *recs, int32_t *status, cudaStream_t stream)
+                             uint4 *recs, int32_t *status, cudaStream_t stream, bool pdl)
 {
     const int64_t rows = pv.hdr->rows_per_layer;
     if (rows == 0) return cudaSuccess;
     PlanDev pd{pv.segs_dev, pv.eps_dev, pv.row_seg_dev, pv.routed_dev, pv.stored_dev, pv.route_tiles_dev};
-    k_row_store<<<dim3((unsigned)((rows + 255) / 256), L), 256, 0, stream>>>(pd, rows, idx, idx_per_layer,
-                                                                            write_identity, recs, status);
+    const dim3 grid((unsigned)((rows + 255) / 256), L);
+    cudaError_t err;
+    if (pdl) {
+        err = launch_pdl(k_row_store, grid, dim3(256), 0, stream, pd, rows, idx, idx_per_layer, write_identity, recs,
+                         status);
+    } else {
+        k_row_store<<<grid, 256, 0, stream>>>(pd, rows, idx, idx_per_layer, write_identity, recs, status);
+        err = cudaGetLastError();
+    }
     count_launches(1);
-    return cudaGetLastError();
+    return err;
 }
 
 }  // namespace rs

@@ -42,6 +42,7 @@ k_lang_pool_v8(const __nv_bfloat16 *__restrict__ h, const rolesub_episode *__res
                int d, float *__restrict__ ctx)
 {
     __shared__ float part[kPoolParts - 1][64][9];
+    pdl_trigger();
     const int l = blockIdx.z, e = blockIdx.y;
     const int cl = threadIdx.x & 63, p = threadIdx.x >> 6;
     const int c8 = blockIdx.x * 64 + cl;
@@ -215,6 +216,8 @@ k_lang_bias_gemv(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__
 {
     const int l = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int f = blockIdx.x * 8 + warp;
+    pdl_trigger();
+    pdl_wait();   // ctx comes from the pooling kernel
     if (f >= F) return;
     const uint4 *w = reinterpret_cast<const uint4 *>(W1 + ((size_t)l * F + f) * (size_t)(2 * d + C) + d + C);
     const float4 *c4 = reinterpret_cast<const float4 *>(ctx + (size_t)l * E * d);
@@ -299,6 +302,8 @@ k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ 
     __shared__ __align__(128) uint8_t sm[3 * BE * BK * 2];   // A hi, A lo, B; later rank 1's sums
     const uint32_t sA0 = static_cast<uint32_t>(__cvta_generic_to_shared(sm));
     const uint32_t sA1 = sA0 + BE * BK * 2, sBs = sA1 + BE * BK * 2;
+    pdl_trigger();
+    pdl_wait();   // ctx comes from the pooling kernel
     const int l = blockIdx.z, tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const uint32_t rank = cluster_rank();
     const int f0 = (blockIdx.x / kSplit) * BF, e0 = blockIdx.y * BE;
@@ -589,17 +594,21 @@ static cudaError_t launch_router_t(const CompressArgs &a)
     cudaError_t err = launch_lang_pool(a);
     if (err != cudaSuccess) return err;
     if (sizeof(T) == 2 && E <= kGemvEpisodes && d % 8 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
-        k_lang_bias_gemv<<<dim3((F + 7) / 8, L), 256, 0, a.stream>>>(
-            (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+        err = launch_pdl(k_lang_bias_gemv, dim3((F + 7) / 8, L), dim3(256), 0, a.stream,
+                         (const __nv_bfloat16 *)a.W1, a.b1, (const float *)a.ws.lang_ctx, E, d, C, F, a.alpha_lang,
+                         a.ws.lang_bias);
     else if (sizeof(T) == 2 && d % 512 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
-        k_lang_bias_mma<8><<<dim3((F + 63) / 64 * 8, (E + 63) / 64, L), 128, 0, a.stream>>>(
-            (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+        err = launch_pdl(k_lang_bias_mma<8>, dim3((F + 63) / 64 * 8, (E + 63) / 64, L), dim3(128), 0, a.stream,
+                         (const __nv_bfloat16 *)a.W1, a.b1, (const float *)a.ws.lang_ctx, E, d, C, F, a.alpha_lang,
+                         a.ws.lang_bias);
     else if (sizeof(T) == 2 && d % 128 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
-        k_lang_bias_mma<2><<<dim3((F + 63) / 64 * 2, (E + 63) / 64, L), 128, 0, a.stream>>>(
-            (const __nv_bfloat16 *)a.W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+        err = launch_pdl(k_lang_bias_mma<2>, dim3((F + 63) / 64 * 2, (E + 63) / 64, L), dim3(128), 0, a.stream,
+                         (const __nv_bfloat16 *)a.W1, a.b1, (const float *)a.ws.lang_ctx, E, d, C, F, a.alpha_lang,
+                         a.ws.lang_bias);
     else
         k_lang_bias<T><<<dim3((F + 31) / 32 * kBiasSplit, (E + 63) / 64, L), 256, 0, a.stream>>>(
             W1, a.b1, a.ws.lang_ctx, E, d, C, F, a.alpha_lang, a.ws.lang_bias);
+    if (err != cudaSuccess) return err;
     if (router_tc_supported(a.shape)) {
         count_launches(1);
         cudaError_t e = cudaGetLastError();

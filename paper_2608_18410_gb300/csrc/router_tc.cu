@@ -90,6 +90,7 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int nkb = d / 64;
     const int total = tiles * L;   // work items (layer, tile), layer-major
+    pdl_trigger();
 
     const uint32_t bar_full = sb + kOffBar;                  // [kStages]
     const uint32_t bar_empty = bar_full + 8 * kStages;       // [kStages]
@@ -237,6 +238,9 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
         const uint32_t lane_base = tmem + ((uint32_t)(32 * quad) << 16);
         const uint32_t swz = (uint32_t)(row & 7);
         float *xch = reinterpret_cast<float *>(sp + kOffXch);
+        // beta comes from the language-bias kernel, which may still run
+        // while the first products do
+        pdl_wait();
         // every epilogue thread walks all of its CTA's items (a wait that
         // gives up returns at once afterwards), so the pairs' named barriers
         // always match
@@ -443,11 +447,14 @@ cudaError_t launch_router_tc(const CompressArgs &a)
     const unsigned grid = (unsigned)(total < sms ? total : sms);
     PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev,
                a.plan.route_tiles_dev};
-    k_router_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(
-        th, tw1, twre, tw2, pd, (int)P.num_route_tiles, L, rows, d, P.num_episodes, S.num_groups, a.b_re,
-        a.ws.lang_bias, a.b2, a.alpha_role, a.idx, P.idx_bytes_per_layer, a.ws.status);
+    // launched as a dependent of the language-bias kernel: the mainloop
+    // reads only caller inputs, the epilogue waits for beta
+    err = launch_pdl(k_router_tc, dim3(grid), dim3(kThreads), kSmemBytes, a.stream, th, tw1, twre, tw2, pd,
+                     (int)P.num_route_tiles, L, rows, d, (int)P.num_episodes, (int)S.num_groups, (const float *)a.b_re,
+                     (const float *)a.ws.lang_bias, (const float *)a.b2, a.alpha_role, a.idx,
+                     (int64_t)P.idx_bytes_per_layer, a.ws.status);
     count_launches(1);
-    return cudaGetLastError();
+    return err;
 }
 
 }  // namespace rs
