@@ -10,13 +10,15 @@
 // group of d_s = 8 values becomes one 16-byte bf16 store into
 // packed[seg][h][i][j][:]. Segments with k = S also get indices 0..S-1.
 //
-// One CTA per (head, layer, range of 128-row tiles), 192 threads:
-//   warp 4  TMA producer: R_h once, then value tiles into a 4-stage ring
+// Persistent: one CTA per SM walks the items (head, layer, range of 128-row
+// tiles), 192 threads:
+//   warp 4  TMA producer: R_h of each item into one of two buffers (the
+//           next item's while this one's tiles are multiplied), value tiles
+//           into a 4-stage ring that runs on across items
 //   warp 5  MMA issuer: one 128x128x128 MMA per tile, TMEM double-buffered
-//   warps 0-3 epilogue: TMEM -> bf16 group stores; the next tile's row
-//           metadata (segment, kept groups) is fetched ahead of time
-// R_h stays in shared memory for the CTA's lifetime, so it is read from
-// L2 once per (head, layer, range) instead of once per tile.
+//   warps 0-3 epilogue: TMEM -> bf16 group stores; the row metadata
+//           (segment, kept groups) is fetched two tiles ahead, across items
+// R_h is read from L2 once per item instead of once per tile.
 #include <cuda.h>
 
 #include "common.cuh"
@@ -36,8 +38,8 @@ constexpr int kDh = 128;
 constexpr int kG = 16;
 constexpr int kStages = 4;
 
-constexpr uint32_t kOffR = 0;                       // R_h: 2 x 16K (MN-blocks)
-constexpr uint32_t kOffV = 32768;                   // V ring: 4 x 32K
+constexpr uint32_t kOffR = 0;                       // R_h: 2 buffers x (2 x 16K MN-blocks)
+constexpr uint32_t kOffV = 65536;                   // V ring: 4 x 32K
 constexpr uint32_t kVBytes = 32768;
 constexpr uint32_t kOffZ = kOffV + kStages * kVBytes;   // bf16 z rows: 128 x 256 B
 constexpr uint32_t kOffBar = kOffZ + 32768;
@@ -86,9 +88,23 @@ k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_p
                                              ((uint32_t)kk << 27) | (uint32_t)((int64_t)sg.n_tokens * k));
 }
 
+struct RotItem {
+    int h, l, t0, nt;
+};
+
+__device__ __forceinline__ RotItem rot_item(int it, int H, int L, int per, int ntiles)
+{
+    RotItem r;
+    r.h = it % H;
+    r.l = (it / H) % L;
+    r.t0 = (it / (H * L)) * per;
+    r.nt = min(per, ntiles - r.t0);
+    return r;
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
 k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_r,
-            const uint4 *__restrict__ meta, int64_t rows, int H, int tiles_per_cta, int ntiles,
+            const uint4 *__restrict__ meta, int64_t rows, int H, int L, int per, int ntiles, int nitems,
             bf16 *__restrict__ packed, int64_t packed_per_layer, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -97,20 +113,20 @@ k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CU
     const uint32_t sraw = smem_u32(smem_raw);
     const uint32_t sb = (sraw + 1023u) & ~1023u;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-    const int h = blockIdx.x, l = blockIdx.y;
-    const int t0 = blockIdx.z * tiles_per_cta;
-    const int nt = min(tiles_per_cta, ntiles - t0);
-    if (nt <= 0) return;
 
-    const uint32_t bar_r = sb + kOffBar;
-    const uint32_t bar_full = bar_r + 8;                 // [4]
+    const uint32_t bar_rfull = sb + kOffBar;             // [2]
+    const uint32_t bar_rempty = bar_rfull + 16;          // [2]
+    const uint32_t bar_full = bar_rempty + 16;           // [4]
     const uint32_t bar_empty = bar_full + 32;            // [4]
     const uint32_t bar_tfull = bar_empty + 32;           // [2]
     const uint32_t bar_tempty = bar_tfull + 16;          // [2]
 
     if (tid == 0) {
         abort_flag = 0;
-        mbar_init(bar_r, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar_rfull + 8 * i, 1);
+            mbar_init(bar_rempty + 8 * i, 1);
+        }
         for (int i = 0; i < kStages; ++i) {
             mbar_init(bar_full + 8 * i, 1);
             mbar_init(bar_empty + 8 * i, 1);
@@ -135,36 +151,59 @@ k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CU
         if (lane == 0) {
             prefetch_tmap(&tm_v);
             prefetch_tmap(&tm_r);
-            mbar_expect_tx(bar_r, 32768);
-            tma_load_3d(sb + kOffR, &tm_r, 0, 0, l * H + h, bar_r);
-            tma_load_3d(sb + kOffR + 16384, &tm_r, 64, 0, l * H + h, bar_r);
-            for (int t = 0; t < nt; ++t) {
-                const int s = t % kStages;
-                if (t >= kStages && !mbar_wait(bar_empty + 8 * s, ((t / kStages) - 1) & 1, status, &abort_flag, 30))
+            bool ok = true;
+            uint32_t gt = 0;   // tiles issued so far (ring position)
+            for (int it = blockIdx.x, n = 0; it < nitems && ok; it += gridDim.x, ++n) {
+                const RotItem w = rot_item(it, H, L, per, ntiles);
+                const uint32_t rb = (uint32_t)n & 1u;
+                // R buffer rb is free once the products of item n - 2 are done
+                if (n >= 2 && !mbar_wait(bar_rempty + 8 * rb, ((uint32_t)(n - 2) >> 1) & 1u, status, &abort_flag, 35))
                     break;
-                const uint32_t st = sb + kOffV + kVBytes * s;
-                const int r0 = (t0 + t) * kRows;
-                mbar_expect_tx(bar_full + 8 * s, kVBytes);
-                tma_load_4d(st, &tm_v, 0, h, r0, l, bar_full + 8 * s);
-                tma_load_4d(st + 16384, &tm_v, 64, h, r0, l, bar_full + 8 * s);
+                mbar_expect_tx(bar_rfull + 8 * rb, 32768);
+                tma_load_3d(sb + kOffR + 32768u * rb, &tm_r, 0, 0, w.l * H + w.h, bar_rfull + 8 * rb);
+                tma_load_3d(sb + kOffR + 32768u * rb + 16384u, &tm_r, 64, 0, w.l * H + w.h, bar_rfull + 8 * rb);
+                for (int t = 0; t < w.nt; ++t, ++gt) {
+                    const uint32_t s = gt % kStages;
+                    if (gt >= kStages &&
+                        !mbar_wait(bar_empty + 8 * s, ((gt / kStages) - 1) & 1, status, &abort_flag, 30)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t st = sb + kOffV + kVBytes * s;
+                    const int r0 = (w.t0 + t) * kRows;
+                    mbar_expect_tx(bar_full + 8 * s, kVBytes);
+                    tma_load_4d(st, &tm_v, 0, w.h, r0, w.l, bar_full + 8 * s);
+                    tma_load_4d(st + 16384, &tm_v, 64, w.h, r0, w.l, bar_full + 8 * s);
+                }
             }
         }
     } else if (warp == 5) {
-        if (lane == 0 && mbar_wait(bar_r, 0, status, &abort_flag, 31)) {
-            for (int t = 0; t < nt; ++t) {
-                const int s = t % kStages, b = t & 1;
-                if (!mbar_wait(bar_full + 8 * s, (t / kStages) & 1, status, &abort_flag, 32)) break;
-                if (t >= 2 && !mbar_wait(bar_tempty + 8 * b, ((t >> 1) - 1) & 1, status, &abort_flag, 33)) break;
-                tc_fence_after();
-                const uint32_t st = sb + kOffV + kVBytes * s;
+        if (lane == 0) {
+            bool ok = true;
+            uint32_t gt = 0;
+            for (int it = blockIdx.x, n = 0; it < nitems && ok; it += gridDim.x, ++n) {
+                const RotItem w = rot_item(it, H, L, per, ntiles);
+                const uint32_t rb = (uint32_t)n & 1u;
+                if (!mbar_wait(bar_rfull + 8 * rb, ((uint32_t)n >> 1) & 1u, status, &abort_flag, 31)) break;
+                for (int t = 0; t < w.nt; ++t, ++gt) {
+                    const uint32_t s = gt % kStages, b = gt & 1u;
+                    if (!mbar_wait(bar_full + 8 * s, (gt / kStages) & 1, status, &abort_flag, 32) ||
+                        (gt >= 2 && !mbar_wait(bar_tempty + 8 * b, ((gt >> 1) - 1) & 1, status, &abort_flag, 33))) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t st = sb + kOffV + kVBytes * s;
 #pragma unroll
-                for (int kk = 0; kk < 8; ++kk) {
-                    const uint64_t a = sdesc_sw128(st + (kk >> 2) * 16384u + (kk & 3) * 32u, 16, 1024);
-                    const uint64_t bd = sdesc_sw128(sb + kOffR + 2048u * kk, 16384, 1024);
-                    mma_bf16(tmem + 128u * b, a, bd, kIdesc, kk > 0);
+                    for (int kk = 0; kk < 8; ++kk) {
+                        const uint64_t a = sdesc_sw128(st + (kk >> 2) * 16384u + (kk & 3) * 32u, 16, 1024);
+                        const uint64_t bd = sdesc_sw128(sb + kOffR + 32768u * rb + 2048u * kk, 16384, 1024);
+                        mma_bf16(tmem + 128u * b, a, bd, kIdesc, kk > 0);
+                    }
+                    mma_commit(bar_empty + 8 * s);
+                    mma_commit(bar_tfull + 8 * b);
                 }
-                mma_commit(bar_empty + 8 * s);
-                mma_commit(bar_tfull + 8 * b);
+                mma_commit(bar_rempty + 8 * rb);
             }
         }
     } else {
@@ -172,54 +211,70 @@ k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CU
         // the records (and the indices behind them) come from the kernels
         // before this one, which may still run while the first products do
         pdl_wait();
-        // row records of this thread's row in tiles t, t+1 (t+2 is fetched
-        // during tile t, so the load latency hides behind two tiles of work)
-        const uint4 *mrow = meta + (int64_t)l * rows + (int64_t)t0 * kRows + tid;
+        // row record of this thread's row in the tile two ahead, across items
         const uint4 zero4 = make_uint4(0, 0, 0, 0);
-        const int64_t rfirst = (int64_t)t0 * kRows + tid;
-        uint4 m0 = rfirst < rows ? __ldg(mrow) : zero4;
-        uint4 m1 = (nt > 1 && rfirst + kRows < rows) ? __ldg(mrow + kRows) : zero4;
-        bf16 *pl = packed + (int64_t)l * packed_per_layer;
-        for (int t = 0; t < nt; ++t) {
-            const int b = t & 1;
-            const int64_t r2 = rfirst + (int64_t)(t + 2) * kRows;
-            const uint4 m2 = (t + 2 < nt && r2 < rows) ? __ldg(mrow + (int64_t)(t + 2) * kRows) : zero4;
-            mbar_wait(bar_tfull + 8 * b, (t >> 1) & 1, status, &abort_flag, 34);
-            tc_fence_after();
-            __syncwarp();
-            const uint64_t gid = (uint64_t)m0.x | ((uint64_t)m0.y << 32);
-            const int k = abort_flag ? 0 : (int)(m0.w >> 27);
-            uint4 *dst = reinterpret_cast<uint4 *>(pl + ((int64_t)m0.z + (int64_t)h * (int64_t)(m0.w & 0x7FFFFFFu)) * 8);
-            // the row's z as 16 bf16 chunks (one per group) in shared memory,
-            // chunk c at position c ^ (row & 15) to spread banks
-            const uint32_t zrow = sb + kOffZ + (uint32_t)tid * 256u;
-            const uint32_t sw = (uint32_t)(tid & 15);
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                uint32_t sa[32], sc[32];
-                tmem_ld32(lane_base + 128u * b + 64u * half, sa);
-                tmem_ld32(lane_base + 128u * b + 64u * half + 32u, sc);
-                tmem_wait_ld();
-#pragma unroll
-                for (int c = 0; c < 8; ++c) {
-                    const uint32_t(&src)[32] = c < 4 ? sa : sc;
-                    const int o = 8 * (c & 3);
-                    st_shared_v4(zrow + ((((uint32_t)(8 * half + c)) ^ sw) << 4),
-                                 pack_bf16(__uint_as_float(src[o]), __uint_as_float(src[o + 1])),
-                                 pack_bf16(__uint_as_float(src[o + 2]), __uint_as_float(src[o + 3])),
-                                 pack_bf16(__uint_as_float(src[o + 4]), __uint_as_float(src[o + 5])),
-                                 pack_bf16(__uint_as_float(src[o + 6]), __uint_as_float(src[o + 7])));
+        int ai = blockIdx.x, at = 0;   // lookahead cursor (item, tile)
+        RotItem aw = ai < nitems ? rot_item(ai, H, L, per, ntiles) : RotItem{0, 0, 0, 0};
+        auto fetch_adv = [&]() -> uint4 {
+            uint4 m = zero4;
+            if (ai < nitems) {
+                const int64_t r = (int64_t)(aw.t0 + at) * kRows + tid;
+                if (r < rows) m = __ldg(meta + (int64_t)aw.l * rows + r);
+                if (++at >= aw.nt) {
+                    at = 0;
+                    ai += gridDim.x;
+                    if (ai < nitems) aw = rot_item(ai, H, L, per, ntiles);
                 }
             }
-            tc_fence_before();
-            mbar_arrive(bar_tempty + 8 * b);   // TMEM buffer b is free for tile t + 2
-            // kept groups in storage order: same-thread shared-memory round trip
-            for (int s = 0; s < k; ++s) {
-                const uint32_t g = (uint32_t)(gid >> (4 * s)) & 15u;
-                dst[s] = ld_shared_v4(zrow + ((g ^ sw) << 4));
+            return m;
+        };
+        uint4 m0 = fetch_adv();
+        uint4 m1 = fetch_adv();
+        const uint32_t zrow = sb + kOffZ + (uint32_t)tid * 256u;
+        const uint32_t sw = (uint32_t)(tid & 15);
+        uint32_t gt = 0;
+        for (int it = blockIdx.x; it < nitems; it += gridDim.x) {
+            const RotItem w = rot_item(it, H, L, per, ntiles);
+            bf16 *pl = packed + (int64_t)w.l * packed_per_layer;
+            for (int t = 0; t < w.nt; ++t, ++gt) {
+                const uint32_t b = gt & 1u;
+                const uint4 m2 = fetch_adv();
+                mbar_wait(bar_tfull + 8 * b, (gt >> 1) & 1, status, &abort_flag, 34);
+                tc_fence_after();
+                __syncwarp();
+                const uint64_t gid = (uint64_t)m0.x | ((uint64_t)m0.y << 32);
+                const int k = abort_flag ? 0 : (int)(m0.w >> 27);
+                uint4 *dst =
+                    reinterpret_cast<uint4 *>(pl + ((int64_t)m0.z + (int64_t)w.h * (int64_t)(m0.w & 0x7FFFFFFu)) * 8);
+                // the row's z as 16 bf16 chunks (one per group) in shared
+                // memory, chunk c at position c ^ (row & 15) to spread banks
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    uint32_t sa[32], sc[32];
+                    tmem_ld32(lane_base + 128u * b + 64u * half, sa);
+                    tmem_ld32(lane_base + 128u * b + 64u * half + 32u, sc);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const uint32_t(&src)[32] = c < 4 ? sa : sc;
+                        const int o = 8 * (c & 3);
+                        st_shared_v4(zrow + ((((uint32_t)(8 * half + c)) ^ sw) << 4),
+                                     pack_bf16(__uint_as_float(src[o]), __uint_as_float(src[o + 1])),
+                                     pack_bf16(__uint_as_float(src[o + 2]), __uint_as_float(src[o + 3])),
+                                     pack_bf16(__uint_as_float(src[o + 4]), __uint_as_float(src[o + 5])),
+                                     pack_bf16(__uint_as_float(src[o + 6]), __uint_as_float(src[o + 7])));
+                    }
+                }
+                tc_fence_before();
+                mbar_arrive(bar_tempty + 8 * b);   // TMEM buffer b is free for the tile two on
+                // kept groups in storage order: same-thread shared-memory round trip
+                for (int s2 = 0; s2 < k; ++s2) {
+                    const uint32_t g = (uint32_t)(gid >> (4 * s2)) & 15u;
+                    dst[s2] = ld_shared_v4(zrow + ((g ^ sw) << 4));
+                }
+                m0 = m1;
+                m1 = m2;
             }
-            m0 = m1;
-            m1 = m2;
         }
     }
     tc_fence_before();
@@ -260,23 +315,30 @@ cudaError_t launch_rotate_tc(const CompressArgs &a)
     cudaError_t err = cudaFuncSetAttribute(k_rotate_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (err != cudaSuccess) return err;
     const int ntiles = (int)((rows + kRows - 1) / kRows);
-    // split each (head, layer) tile list so that there are at least ~4 CTAs per SM-wave
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0)
+        sms = 152;
+    // split each (head, layer) tile list until there are at least eight
+    // items per persistent CTA, so that the last round of items is short
     int splits = 1;
-    while ((int64_t)H * L * splits < 4 * 152 && splits < ntiles) ++splits;
+    while ((int64_t)H * L * splits < 8 * (int64_t)sms && splits < ntiles) ++splits;
     const int per = (ntiles + splits - 1) / splits;
     splits = (ntiles + per - 1) / per;
+    const int nitems = H * L * splits;
+    const unsigned grid = (unsigned)(nitems < sms ? nitems : sms);
     uint4 *meta = reinterpret_cast<uint4 *>(a.ws.row_store);
     if (!a.records_ready) {
         // the records and then the products start while the router's tail
         // still runs; both wait for their predecessor before reading its output
         err = launch_row_store(a.plan, L, a.idx, P.idx_bytes_per_layer, true, meta, a.ws.status, a.stream, true);
         if (err != cudaSuccess) return err;
-        err = launch_pdl(k_rotate_tc, dim3(H, L, splits), dim3(kThreads), kSmemBytes, a.stream, tv, tr,
-                         (const uint4 *)meta, rows, H, per, ntiles, (bf16 *)a.packed,
-                         (int64_t)P.packed_elems_per_layer, a.ws.status);
+        err = launch_pdl(k_rotate_tc, dim3(grid), dim3(kThreads), kSmemBytes, a.stream, tv, tr, (const uint4 *)meta,
+                         rows, H, L, per, ntiles, nitems, (bf16 *)a.packed, (int64_t)P.packed_elems_per_layer,
+                         a.ws.status);
     } else {
-        k_rotate_tc<<<dim3(H, L, splits), kThreads, kSmemBytes, a.stream>>>(
-            tv, tr, meta, rows, H, per, ntiles, (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
+        k_rotate_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(tv, tr, meta, rows, H, L, per, ntiles, nitems,
+                                                             (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
         err = cudaGetLastError();
     }
     count_launches(1);
