@@ -87,6 +87,8 @@ k_budget_select(PlanDev plan, int64_t rows, const float *__restrict__ scores, ui
     __shared__ int part[kBT];
     __shared__ int sh_c;
     __shared__ long long sh_left;
+    pdl_trigger();
+    pdl_wait();   // the scores come from the router kernel just before
     const int tid = threadIdx.x, l = blockIdx.y;
     const rolesub_segment sg = plan.segs[blockIdx.x];
     const int n = sg.n_tokens, km = sg.k;
@@ -199,6 +201,7 @@ k_row_store_budget(PlanDev plan, int64_t rows, const uint8_t *__restrict__ idx, 
 {
     extern __shared__ __align__(16) uint8_t smb[];
     __shared__ int part[kBT];
+    pdl_trigger();
     const int tid = threadIdx.x, l = blockIdx.y;
     const rolesub_segment sg = plan.segs[blockIdx.x];
     const int n = sg.n_tokens;
@@ -259,11 +262,11 @@ cudaError_t launch_budget_select(const CompressArgs &a, const float *scores, uin
     if (err != cudaSuccess) return err;
     const PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev,
                      a.plan.route_tiles_dev};
-    k_budget_select<<<dim3((unsigned)P.num_segments, a.shape->num_layers), kBT, smem, a.stream>>>(
-        pd, P.rows_per_layer, scores, a.idx, P.idx_bytes_per_layer, k_tok,
-        reinterpret_cast<uint4 *>(a.ws.row_store));
+    err = launch_pdl(k_budget_select, dim3((unsigned)P.num_segments, a.shape->num_layers), dim3(kBT), smem, a.stream,
+                     pd, (int64_t)P.rows_per_layer, scores, a.idx, (int64_t)P.idx_bytes_per_layer, k_tok,
+                     reinterpret_cast<uint4 *>(a.ws.row_store));
     count_launches(1);
-    return cudaGetLastError();
+    return err;
 }
 
 cudaError_t launch_row_store_budget(const PlanView &pv, int L, const uint8_t *idx, int64_t idx_per_layer,

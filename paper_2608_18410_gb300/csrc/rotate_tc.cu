@@ -328,19 +328,15 @@ cudaError_t launch_rotate_tc(const CompressArgs &a)
     const int nitems = H * L * splits;
     const unsigned grid = (unsigned)(nitems < sms ? nitems : sms);
     uint4 *meta = reinterpret_cast<uint4 *>(a.ws.row_store);
+    // the records (when built here) and then the products start while the
+    // router's tail still runs; both wait for their predecessor before
+    // reading its output
     if (!a.records_ready) {
-        // the records and then the products start while the router's tail
-        // still runs; both wait for their predecessor before reading its output
         err = launch_row_store(a.plan, L, a.idx, P.idx_bytes_per_layer, true, meta, a.ws.status, a.stream, true);
         if (err != cudaSuccess) return err;
-        err = launch_pdl(k_rotate_tc, dim3(grid), dim3(kThreads), kSmemBytes, a.stream, tv, tr, (const uint4 *)meta,
-                         rows, H, L, per, ntiles, nitems, (bf16 *)a.packed, (int64_t)P.packed_elems_per_layer,
-                         a.ws.status);
-    } else {
-        k_rotate_tc<<<grid, kThreads, kSmemBytes, a.stream>>>(tv, tr, meta, rows, H, L, per, ntiles, nitems,
-                                                             (bf16 *)a.packed, P.packed_elems_per_layer, a.ws.status);
-        err = cudaGetLastError();
     }
+    err = launch_pdl(k_rotate_tc, dim3(grid), dim3(kThreads), kSmemBytes, a.stream, tv, tr, (const uint4 *)meta, rows,
+                     H, L, per, ntiles, nitems, (bf16 *)a.packed, (int64_t)P.packed_elems_per_layer, a.ws.status);
     count_launches(1);
     return err;
 }

@@ -223,7 +223,7 @@ k_lang_bias_gemv(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__
     const float4 *c4 = reinterpret_cast<const float4 *>(ctx + (size_t)l * E * d);
     const int n8 = d / 8;
     float acc[kGemvEpisodes] = {};
-#pragma unroll 4
+#pragma unroll 8
     for (int k8 = lane; k8 < n8; k8 += 32) {
         const uint4 wv = __ldg(w + k8);
         const __nv_bfloat162 *wp = reinterpret_cast<const __nv_bfloat162 *>(&wv);

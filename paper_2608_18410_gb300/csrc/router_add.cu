@@ -44,6 +44,8 @@ k_lang_term_add(const T *__restrict__ W_l, const float *__restrict__ b_l, const 
 {
     const int l = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int item = blockIdx.x * 8 + warp;
+    pdl_trigger();
+    pdl_wait();   // ctx comes from the pooling kernel
     if (item >= E * G) return;
     const int e = item / G, s = item % G;
     const T *w = W_l + ((size_t)l * G + s) * d;
@@ -66,6 +68,8 @@ k_lang_term_add4(const T *__restrict__ W_l, const float *__restrict__ b_l, const
 {
     __shared__ float part[8][kTermEp * kTermMaxG];
     const int l = blockIdx.y, e0 = blockIdx.x * kTermEp, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    pdl_trigger();
+    pdl_wait();   // ctx comes from the pooling kernel
     float acc[kTermEp][kTermMaxG];
 #pragma unroll
     for (int i = 0; i < kTermEp; ++i)
@@ -208,6 +212,7 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
     const uint32_t bar_full = sb + off_bar, bar_empty = bar_full + 8u * kTMaxStages,
                    bar_acc = bar_empty + 8u * kTMaxStages;
     const uint32_t ncols = tmem_cols_for(nb);
+    pdl_trigger();
 
     if (tid == 0) {
         abort_flag = 0;
@@ -283,6 +288,9 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
         }
         const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
         const float *bre = b_re + (size_t)l * C;
+        // the language term comes from the kernel before this one, which may
+        // still run while the products do
+        pdl_wait();
         mbar_wait(bar_acc, 0, status, &abort_flag, 42);
         tc_fence_after();
         __syncwarp();
@@ -392,13 +400,15 @@ cudaError_t launch_additive_t(const CompressArgs &a, const AdditiveWeights &w)
     cudaError_t err = launch_lang_pool(a);
     if (err != cudaSuccess) return err;
     if (G <= kTermMaxG)
-        k_lang_term_add4<T><<<dim3((unsigned)((E + kTermEp - 1) / kTermEp), L), 256, 0, a.stream>>>(
-            (const T *)w.W_l, w.b_l, a.ws.lang_ctx, E, d, G, a.alpha_lang, a.ws.lang_bias);
+        err = launch_pdl(k_lang_term_add4<T>, dim3((unsigned)((E + kTermEp - 1) / kTermEp), L), dim3(256), 0,
+                         a.stream, (const T *)w.W_l, w.b_l, (const float *)a.ws.lang_ctx, E, d, G, a.alpha_lang,
+                         a.ws.lang_bias);
     else
-        k_lang_term_add<T><<<dim3((unsigned)((E * G + 7) / 8), L), 256, 0, a.stream>>>(
-            (const T *)w.W_l, w.b_l, a.ws.lang_ctx, E, d, G, a.alpha_lang, a.ws.lang_bias);
+        err = launch_pdl(k_lang_term_add<T>, dim3((unsigned)((E * G + 7) / 8), L), dim3(256), 0, a.stream,
+                         (const T *)w.W_l, w.b_l, (const float *)a.ws.lang_ctx, E, d, G, a.alpha_lang,
+                         a.ws.lang_bias);
     count_launches(1);
-    if ((err = cudaGetLastError()) != cudaSuccess) return err;
+    if (err != cudaSuccess) return err;
     const PlanDev pd{a.plan.segs_dev, a.plan.eps_dev, a.plan.row_seg_dev, a.plan.routed_dev, a.plan.stored_dev,
                      a.plan.route_tiles_dev};
     if (sizeof(T) == 2 && additive_tc_supported(a.shape)) {
@@ -430,11 +440,12 @@ cudaError_t launch_additive_t(const CompressArgs &a, const AdditiveWeights &w)
         }
         err = cudaFuncSetAttribute(k_router_add_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (err != cudaSuccess) return err;
-        k_router_add_tc<<<dim3((unsigned)P.num_route_tiles, L), kTThreads, smem, a.stream>>>(
-            th, twv, twre, pd, rows, d, C, E, nb, stages, w.b_v, a.b_re, (const bf16 *)w.W_role, a.ws.lang_bias,
-            a.alpha_role, a.idx, P.idx_bytes_per_layer, w.u, w.scores, a.ws.status);
+        err = launch_pdl(k_router_add_tc, dim3((unsigned)P.num_route_tiles, L), dim3(kTThreads), smem, a.stream, th,
+                         twv, twre, pd, rows, d, C, E, nb, stages, w.b_v, a.b_re, (const bf16 *)w.W_role,
+                         (const float *)a.ws.lang_bias, a.alpha_role, a.idx, (int64_t)P.idx_bytes_per_layer, w.u,
+                         w.scores, a.ws.status);
         count_launches(1);
-        return cudaGetLastError();
+        return err;
     }
     if (w.scores) return cudaErrorInvalidValue;   // score mode: tensor-core path only
     const size_t smem = (size_t)8 * (G + C) * sizeof(float);
