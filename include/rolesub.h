@@ -26,7 +26,12 @@
  *    rolesub_status. Device work is enqueued on the caller's CUDA stream
  *    (cudaStream_t passed as void*; NULL = legacy default stream) and is
  *    asynchronous; no entry point synchronises except
- *    rolesub_get_device_status.
+ *    rolesub_get_device_status. The first kernel of a call starts after
+ *    all earlier work on the stream; the later kernels of the same call are
+ *    launched as programmatic dependents of the kernel before them (they
+ *    may be scheduled while it finishes and wait for it before reading
+ *    anything it writes), so a call's result is the same as with plain
+ *    stream order.
  *  - The caller owns every buffer. The library allocates no memory and keeps
  *    no state between calls, apart from one-time per-process lookups and a
  *    diagnostic counter of kernel launches (rolesub_launch_count).
