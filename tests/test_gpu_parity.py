@@ -194,12 +194,24 @@ def test_repeated_calls_are_deterministic():
 @pytest.mark.parametrize("H", [1, 3, 5])
 def test_tensor_core_router_short_hidden(H):
     """The tensor-core router (F = 256, C = 64, S = 16) with d = 128, 384 and
-    640: main loops of 2, 6 and 10 blocks, so the ring's last stages are
-    unused or partly used when the epilogue weights are loaded into them."""
+    640: main loops of 2, 6 and 10 blocks, so the ring wraps a different
+    number of times before the epilogue weights go into stage 0."""
     E = synth.Episode
     wl = synth.Workload(f"tc_router_h{H}", "bf16", L=2, H=H, dh=128, G=16, C=64, F=256,
                         episodes=(E(140, 20, 64, 3, 6), E(9, 40, 5, 8, 16)), seed=14)
     _run(wl, [(l, e) for l in range(2) for e in range(2)])
+
+
+@pytest.mark.parametrize("L", [151, 153])
+def test_persistent_kernels_uneven_item_counts(L):
+    """One 128-row router tile per layer: with 152 SMs, L = 151 leaves one
+    persistent router CTA without work and L = 153 gives one CTA a second
+    item (a second trip round the ring, TMEM and barrier phases); the
+    rotation's (head, layer, tile range) items wrap unevenly over its CTAs."""
+    E = synth.Episode
+    wl = synth.Workload(f"persist_l{L}", "bf16", L=L, H=2, dh=128, G=16, C=64, F=256,
+                        episodes=(E(128, 8, 16, 4, 16),), seed=16)
+    _run(wl, [(0, 0), (L // 2, 0), (L - 2, 0), (L - 1, 0)])
 
 
 def test_attention_split_over_launches():
