@@ -33,8 +33,10 @@
  *    anything it writes), so a call's result is the same as with plain
  *    stream order.
  *  - The caller owns every buffer. The library allocates no memory and keeps
- *    no state between calls, apart from one-time per-process lookups and a
- *    diagnostic counter of kernel launches (rolesub_launch_count).
+ *    no state between calls, apart from one-time per-process lookups, a
+ *    diagnostic counter of kernel launches (rolesub_launch_count) and the
+ *    fixed per-GPU scratch array of rolesub_compress_static, which that
+ *    call alone uses and which keeps its contents from one call to the next.
  *  - Device pointers must be 16-byte aligned; ROLESUB_EINVAL otherwise.
  *  - Argument errors return ROLESUB_EINVAL (or ROLESUB_EUNSUPPORTED for a
  *    valid geometry this build does not implement) before anything is
@@ -380,6 +382,26 @@ rolesub_status rolesub_attend_dense(const rolesub_shape *shape, const void *plan
 rolesub_status rolesub_get_device_status(const void *workspace, void *stream, int32_t *code_out,
                                          int32_t *detail_out);
 
+/*
+ * Self-test of the bounded in-kernel waits (the library's failure handling;
+ * the paper has no counterpart). Launches one small kernel in which one
+ * thread waits on an mbarrier that nothing arrives on, through the same wait
+ * loop the tensor-core kernels use but with a limit of limit_ns, and a
+ * second thread waits on it with the production limit (about 2 s). The
+ * first wait runs out: it records ROLESUB_ETIMEOUT with site 900 in the
+ * workspace's status word and raises the CTA's abort flag, which ends the
+ * second wait at once (it records nothing). No copy or tensor-core work is
+ * in flight; the kernel then returns and the context stays usable.
+ *   limit_ns   1e3 .. 2e9
+ *   workspace  device, 16-byte aligned, at least 256 bytes; its status word
+ *              should be clear before the call
+ *   out        device int64[4], 16-byte aligned: {first wait completed (0/1),
+ *              its duration in ns, second wait completed (0/1), its duration}
+ * ROLESUB_EINVAL (nothing launched) on bad arguments, ROLESUB_ECUDA on a
+ * failed launch.
+ */
+rolesub_status rolesub_wait_selftest(int64_t limit_ns, void *workspace, int64_t *out, void *stream);
+
 /* Enqueues a clear of the status word on the stream. */
 rolesub_status rolesub_reset_device_status(void *workspace, void *stream);
 
@@ -414,9 +436,10 @@ int32_t rolesub_version(void);
  *    call clears what must start at zero itself. Calls whose work overlaps
  *    on the GPU (different streams, or different host threads on one
  *    device) race on the array: serialise them.
- *  - The device status word is kept in the array and is not readable by
- *    the caller; the compress kernels only report stored indices >= S,
- *    which the router does not produce.
+ *  - The device status word (a wait in the router or rotation kernel that
+ *    ran out, ROLESUB_ETIMEOUT, with the site in the detail) is kept at the
+ *    start of the array. Each call clears it when it starts; read the
+ *    status of the latest call with rolesub_static_device_status.
  * Other arguments, errors and results: as rolesub_compress.
  */
 #define ROLESUB_STATIC_SCRATCH_BYTES (8u << 20)
@@ -426,6 +449,17 @@ rolesub_status rolesub_compress_static(const rolesub_shape *shape, const void *p
                                        const void *W1, const float *b1, const void *W2,
                                        const float *b2, float alpha_role, float alpha_lang,
                                        void *packed_v, uint8_t *idx, void *stream);
+
+/* Waits for the stream, then reads the status word that the latest
+ * rolesub_compress_static call on the current device left in the fixed
+ * array: *code_out = 0 when no kernel reported a problem, else a ROLESUB_E*
+ * code; *detail_out (may be NULL) receives the reported site or item. No
+ * counterpart in the paper. Allocates nothing; like the static call, its
+ * first use on a device looks up the array's address. */
+rolesub_status rolesub_static_device_status(void *stream, int32_t *code_out, int32_t *detail_out);
+
+/* ROLESUB_STATIC_SCRATCH_BYTES as compiled into the loaded library. */
+size_t rolesub_static_scratch_bytes(void);
 
 /* Number of kernels this process has launched through the library so far
  * (all threads, all devices). Diagnostic only: a caller takes the

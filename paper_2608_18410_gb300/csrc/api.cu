@@ -810,3 +810,21 @@ extern "C" rolesub_status rolesub_compress_static(
     if (rs::launch_router(a) != cudaSuccess) return ROLESUB_ECUDA;
     return from_cuda(rs::launch_rotate_pack(a));
 }
+
+extern "C" rolesub_status rolesub_static_device_status(void *stream, int32_t *code_out, int32_t *detail_out)
+{
+    if (!code_out) return ROLESUB_EINVAL;
+    void *scratch = nullptr;
+    rolesub_status st = static_scratch(&scratch);
+    if (st != ROLESUB_OK) return st;
+    // the status word is the first 8 bytes of the array (code, detail)
+    int32_t hs[2] = {0, 0};
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaMemcpyAsync(hs, scratch, sizeof(hs), cudaMemcpyDeviceToHost, s) != cudaSuccess) return ROLESUB_ECUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return ROLESUB_ECUDA;
+    *code_out = hs[0];
+    if (detail_out) *detail_out = hs[1];
+    return ROLESUB_OK;
+}
+
+extern "C" size_t rolesub_static_scratch_bytes(void) { return (size_t)ROLESUB_STATIC_SCRATCH_BYTES; }

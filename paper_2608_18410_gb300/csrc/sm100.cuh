@@ -100,18 +100,26 @@ static __device__ __noinline__ void wait_timed_out(int32_t *status, volatile int
     *abort = 1;
 }
 
-static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int32_t *status,
-                                                   volatile int *abort, int where)
+// The sleeping wait loop: true once the phase completes; false when *abort
+// is raised, or after limit_ns (then the site is recorded and *abort raised).
+__device__ __forceinline__ bool mbar_wait_loop(uint32_t bar, uint32_t parity, int32_t *status,
+                                               volatile int *abort, int where, uint64_t limit_ns)
 {
     const uint64_t t0 = global_ns();
 #pragma unroll 1
     for (;;) {
         if (mbar_try_wait_sleep(bar, parity, kSleepHintNs)) return true;
         if (*abort) return false;
-        if (global_ns() - t0 > kWaitLimitNs) break;
+        if (global_ns() - t0 > limit_ns) break;
     }
     wait_timed_out(status, abort, where);
     return false;
+}
+
+static __device__ __noinline__ bool mbar_wait_slow(uint32_t bar, uint32_t parity, int32_t *status,
+                                                   volatile int *abort, int where)
+{
+    return mbar_wait_loop(bar, parity, status, abort, where, kWaitLimitNs);
 }
 
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, int32_t *status,

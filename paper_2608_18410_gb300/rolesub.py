@@ -33,9 +33,8 @@ EXPORTS = ("rolesub_plan_size", "rolesub_layout_plan", "rolesub_workspace_size",
            "rolesub_launch_count", "rolesub_compress_static", "rolesub_compress_additive",
            "rolesub_budget_workspace_size", "rolesub_compress_budget", "rolesub_attend_budget",
            "rolesub_select_count", "rolesub_select_tokens", "rolesub_dense_workspace_size",
-           "rolesub_compress_dense", "rolesub_attend_dense")
-
-STATIC_SCRATCH_BYTES = 8 << 20
+           "rolesub_compress_dense", "rolesub_attend_dense", "rolesub_static_device_status",
+           "rolesub_static_scratch_bytes", "rolesub_wait_selftest")
 
 
 class RoleSubError(RuntimeError):
@@ -131,9 +130,13 @@ def lib():
                                                                      _vp, ctypes.c_size_t, _vp])
         L.rolesub_launch_count.argtypes = []
         L.rolesub_launch_count.restype = ctypes.c_uint64
+        L.rolesub_static_device_status.argtypes = [_vp, _i32p, _i32p]
+        L.rolesub_wait_selftest.argtypes = [ctypes.c_int64, _vp, _vp, _vp]
+        L.rolesub_static_scratch_bytes.argtypes = []
+        L.rolesub_static_scratch_bytes.restype = ctypes.c_size_t
         for name in EXPORTS:
             if name not in ("rolesub_status_string", "rolesub_version", "rolesub_launch_count",
-                            "rolesub_select_count"):
+                            "rolesub_select_count", "rolesub_static_scratch_bytes"):
                 getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -278,11 +281,26 @@ def rolesub_attend(shape, plan: Plan, plan_dev, q, q_strides, K, k_strides, pack
 def rolesub_compress_static(shape, plan: Plan, plan_dev, h, v, R, W_re, b_re, W1, b1, W2, b2,
                             alpha_role, alpha_lang, packed_v, idx, stream=None):
     """rolesub_compress for callers that cannot allocate: the scratch is the
-    library's fixed per-GPU array (STATIC_SCRATCH_BYTES); no workspace."""
+    library's fixed per-GPU array (rolesub_static_scratch_bytes()); no workspace."""
     _check("rolesub_compress_static", lib().rolesub_compress_static(
         ctypes.byref(shape), plan.host_ptr, _ptr(plan_dev), _ptr(h), _ptr(v), _ptr(R), _ptr(W_re),
         _ptr(b_re), _ptr(W1), _ptr(b1), _ptr(W2), _ptr(b2), float(alpha_role), float(alpha_lang),
         _ptr(packed_v), _ptr(idx), _stream(stream)))
+
+
+def rolesub_static_device_status(stream=None):
+    """(code, detail) of the status word the latest rolesub_compress_static
+    call left in the fixed array (waits for the stream)."""
+    code = ctypes.c_int32(0)
+    detail = ctypes.c_int32(0)
+    _check("rolesub_static_device_status", lib().rolesub_static_device_status(
+        _stream(stream), ctypes.byref(code), ctypes.byref(detail)))
+    return code.value, detail.value
+
+
+def rolesub_static_scratch_bytes():
+    """Size of the fixed scratch array compiled into the loaded library."""
+    return int(lib().rolesub_static_scratch_bytes())
 
 
 def rolesub_select_count(n_view, ratio):
@@ -337,6 +355,13 @@ def rolesub_get_device_status(workspace, stream=None):
 
 def rolesub_reset_device_status(workspace, stream=None):
     _check("rolesub_reset_device_status", lib().rolesub_reset_device_status(_ptr(workspace), _stream(stream)))
+
+
+def rolesub_wait_selftest(limit_ns, workspace, out, stream=None):
+    """Launches the bounded-wait self-test (see the header); out is a device
+    int64 tensor of 4 elements."""
+    _check("rolesub_wait_selftest", lib().rolesub_wait_selftest(
+        int(limit_ns), _ptr(workspace), _ptr(out), _stream(stream)))
 
 
 def rolesub_status_string(code):

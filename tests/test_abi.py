@@ -41,6 +41,13 @@ def test_every_declared_symbol_is_exported(rsm):
     assert rsm.rolesub_status_string(1) == "invalid argument"
 
 
+def test_static_scratch_size_matches_header(rsm):
+    txt = open(os.path.join(ROOT, "include", "rolesub.h")).read()
+    m = re.search(r"#define ROLESUB_STATIC_SCRATCH_BYTES \((\d+)u << (\d+)\)", txt)
+    assert m, "ROLESUB_STATIC_SCRATCH_BYTES not found in the header"
+    assert rsm.rolesub_static_scratch_bytes() == int(m.group(1)) << int(m.group(2))
+
+
 def test_struct_sizes_match_header(rsm):
     assert ctypes.sizeof(rsm.Shape) == 32
     assert ctypes.sizeof(rsm.Segment) == 40
@@ -268,3 +275,13 @@ def test_dense_calls_reject_bad_arguments_before_any_launch(rsm):
           0.0, fake, fake, big, None]
     at[13] = None                       # R_dense
     assert L.rolesub_attend_dense(*at) == 1
+
+
+def test_wait_selftest_rejects_bad_arguments_before_any_launch(rsm):
+    L = rsm.lib()
+    fake = 1 << 20            # never touched: every check comes before the launch
+    assert L.rolesub_wait_selftest(999, fake, fake, None) == 1
+    assert L.rolesub_wait_selftest(2_000_000_001, fake, fake, None) == 1
+    assert L.rolesub_wait_selftest(5_000_000, None, fake, None) == 1
+    assert L.rolesub_wait_selftest(5_000_000, fake, None, None) == 1
+    assert L.rolesub_wait_selftest(5_000_000, fake + 8, fake, None) == 1

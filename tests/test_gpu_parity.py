@@ -202,12 +202,15 @@ def test_tensor_core_router_short_hidden(H):
     _run(wl, [(l, e) for l in range(2) for e in range(2)])
 
 
-@pytest.mark.parametrize("L", [151, 153])
-def test_persistent_kernels_uneven_item_counts(L):
-    """One 128-row router tile per layer: with 152 SMs, L = 151 leaves one
-    persistent router CTA without work and L = 153 gives one CTA a second
-    item (a second trip round the ring, TMEM and barrier phases); the
-    rotation's (head, layer, tile range) items wrap unevenly over its CTAs."""
+@pytest.mark.parametrize("extra", [-1, 1])
+def test_persistent_kernels_uneven_item_counts(extra):
+    """One 128-row router tile per layer, L = (SM count) - 1 or + 1. The
+    persistent router launches min(items, SMs) CTAs, so with one item fewer
+    than SMs every CTA takes exactly one item (the grid shrinks; no CTA is
+    idle), and with one more one CTA takes a second item (a second trip round
+    the ring, TMEM and barrier phases); the rotation's (head, layer, tile
+    range) items wrap unevenly over its CTAs."""
+    L = torch.cuda.get_device_properties(0).multi_processor_count + extra
     E = synth.Episode
     wl = synth.Workload(f"persist_l{L}", "bf16", L=L, H=2, dh=128, G=16, C=64, F=256,
                         episodes=(E(128, 8, 16, 4, 16),), seed=16)

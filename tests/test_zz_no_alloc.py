@@ -6,8 +6,9 @@ library, so it takes no workspace.
 
 The test goes through the C ABI: the allocation-free call must give what
 rolesub_compress gives (same tolerance as the parity tests), on two calls
-in a row (the array keeps the previous call's contents), and must reject a
-problem whose scratch does not fit. This file is collected last so that a
+in a row (the array keeps the previous call's contents), must leave a clean
+status word readable through rolesub_static_device_status, and must reject
+a problem whose scratch does not fit. This file is collected last so that a
 run stopping at the first failure has already run every other test.
 """
 import ctypes
@@ -63,7 +64,7 @@ def test_static_scratch_compress_matches_workspace_compress(make):
     inp = synth.gen_inputs(wl)
     rs = rolesub.RoleSub(wl.L, wl.H, wl.dh, wl.G, wl.C, wl.F, wl.dtype, wl.n_tok_array(), wl.k_array(),
                          wl.n_query_array())
-    assert rs.ws_bytes <= rolesub.STATIC_SCRATCH_BYTES
+    assert rs.ws_bytes <= rolesub.rolesub_static_scratch_bytes()
     d = {k: _dev(v) for k, v in inp.items()}
     args = (d["h"], d["v"], d["R"], d["W_re"], d["b_re"], d["W1"], d["b1"], d["W2"], d["b2"],
             wl.alpha_role, wl.alpha_lang)
@@ -79,6 +80,7 @@ def test_static_scratch_compress_matches_workspace_compress(make):
         torch.cuda.synchronize()
         if call == 1:
             assert torch.cuda.mem_get_info()[0] == free0, "the call must not allocate"
+        assert rolesub.rolesub_static_device_status() == (0, 0), f"call {call}: device status"
         nidx = rs.plan.hdr.idx_bytes_per_layer
         assert torch.equal(i[:, :nidx], ref_i[:, :nidx]), f"call {call}: group indices differ"
         _rows_close(p, ref_p, wl, rs.plan, TOL[wl.dtype])
@@ -89,7 +91,7 @@ def test_static_scratch_rejects_problems_that_do_not_fit():
     wl = synth.c4()
     shape = rolesub.make_shape(wl.L, wl.H, wl.dh, wl.G, wl.C, wl.F, wl.dtype)
     plan = rolesub.Plan(shape, wl.n_tok_array(), wl.k_array(), wl.n_query_array())
-    assert plan.workspace_size() > rolesub.STATIC_SCRATCH_BYTES
+    assert plan.workspace_size() > rolesub.rolesub_static_scratch_bytes()
     fake = 1 << 20            # never touched: the size check comes first
     rc = rolesub.lib().rolesub_compress_static(ctypes.byref(shape), plan.host_ptr, fake, *([fake] * 9),
                                                0.1, 0.1, fake, fake, None)
