@@ -349,15 +349,20 @@ rolesub_status rolesub_select_tokens(int32_t num_episodes, int32_t num_views, in
  * order at packed_off + (i k + j) g (the plan's segment sizes are the same:
  * n k H d_s = n k g).
  *   R_dense [L][d][d] (R[m][n], dtype); other arguments as rolesub_compress.
+ * Only the kept groups are computed: z_s = R_s^T v (R_s the g columns of
+ * group s) for each kept (token, group) pair, written to its packed slot.
  * rolesub_attend_dense: attention over such a cache; every head's output
  * needs all d rotated dims (o_{q,h} = R_h sum_j p_j M_j z_j with R_h the d_h
  * rows of head h), so the call first forms the routed values
- * v~_j = R M_j z_j of every cache row on the tensor core and then attends
+ * v~_j = R M_j z_j = sum over kept s of R_s z_{j,s} of every cache row on
+ * the tensor core (reading the packed groups in place) and then attends
  * over them; arguments as rolesub_attend plus R_dense.
  * workspace: at least rolesub_dense_workspace_size bytes for either call
- * (the common workspace, then 2 L rows d + L H d_h^2 bf16 elements).
- * Supported geometry: bf16, d_h = 128, S = 16, d a multiple of 256;
- * otherwise ROLESUB_EUNSUPPORTED.
+ * (the common workspace, then L rows d + L H d_h^2 bf16 elements, L rows
+ * int32, 2 L idx_bytes_per_layer int32 and 32 L ceil(rows / 4096) int32).
+ * Supported geometry: bf16, d_h = 128, S = 16, d a multiple of 256 with
+ * g = d / 16 equal to 64, 128 or a multiple of 256, and a plan laid out by
+ * rolesub_plan_build; otherwise ROLESUB_EUNSUPPORTED.
  */
 rolesub_status rolesub_dense_workspace_size(const rolesub_shape *shape, const void *plan_host,
                                             size_t *bytes);

@@ -3,6 +3,7 @@
 #include <math.h>
 #include <string.h>
 
+#include <algorithm>
 #include <atomic>
 
 #include "common.cuh"
@@ -134,22 +135,80 @@ Workspace carve(const WsSizes &w, void *base)
 
 rolesub_status from_cuda(cudaError_t e) { return e == cudaSuccess ? ROLESUB_OK : ROLESUB_ECUDA; }
 
-// The dense-rotation path: bf16, d_h = 128, S = 16 (the tensor-core
-// rotation's store records and the tensor-core attention), d % 256 == 0 (the
-// GEMM's column tile).
+// The dense-rotation path: bf16, d_h = 128, S = 16 (the attention kernel
+// reads v~ through store records), d % 256 == 0 (the v~ GEMM's column tile)
+// and g = d / 16 either 64, 128 or a multiple of 256 (a group is a whole
+// number of 64-wide K blocks, and a whole number of N tiles of the z GEMM).
 bool dense_supported(const rolesub_shape *s)
 {
-    const int d = s->num_heads * s->head_dim;
-    return rs::rotate_tc_supported(s) && rs::attend_tc_supported(s) && d % 256 == 0 && d <= 65536;
+    const int d = s->num_heads * s->head_dim, g = d / 16;
+    return rs::rotate_tc_supported(s) && rs::attend_tc_supported(s) && d % 256 == 0 && d <= 65536 &&
+           (g == 64 || g == 128 || g % 256 == 0);
 }
 
-// Z (compress) or M z and v~ (attend), [L][rows][d] bf16 each, and the
-// identity rotations [L][H][d_h][d_h] bf16, after the common workspace.
-size_t dense_extra_bytes(const rolesub_shape *s, const rolesub_plan *p)
+int dense_chunks(const rolesub_plan *p) { return (int)((p->rows_per_layer + rs::kDenseChunk - 1) / rs::kDenseChunk); }
+
+// After the common workspace: v~ [L][rows][d] bf16, perm [L][rows] int32,
+// the identity rotations [L][H][d_h][d_h] bf16, the pair lists [L][idx
+// bytes per layer] int2, and the chunk tables [L][chunks][32] int32.
+struct DenseWs {
+    size_t vt, perm, ident, pairs, meta, total;
+};
+
+DenseWs dense_ws(const rolesub_shape *s, const rolesub_plan *p)
 {
-    const size_t d = (size_t)s->num_heads * s->head_dim, L = s->num_layers;
-    const size_t vals = align_up(2 * L * (size_t)p->rows_per_layer * d, kAlign);
-    return 2 * vals + align_up(2 * L * s->num_heads * (size_t)s->head_dim * s->head_dim, kAlign);
+    const size_t d = (size_t)s->num_heads * s->head_dim, L = s->num_layers, rows = (size_t)p->rows_per_layer;
+    DenseWs w;
+    w.vt = align_up(2 * L * rows * d, kAlign);
+    w.perm = align_up(4 * L * rows, kAlign);
+    w.ident = align_up(2 * L * s->num_heads * (size_t)s->head_dim * s->head_dim, kAlign);
+    w.pairs = align_up(8 * L * (size_t)p->idx_bytes_per_layer, kAlign);
+    w.meta = align_up(4 * L * (size_t)dense_chunks(p) * rs::kDenseMetaStride, kAlign);
+    w.total = w.vt + w.perm + w.ident + w.pairs + w.meta;
+    return w;
+}
+
+size_t dense_extra_bytes(const rolesub_shape *s, const rolesub_plan *p) { return dense_ws(s, p).total; }
+
+// The layout the dense kernels rely on (the one rolesub_plan_build makes):
+// segments in row order, indices and packed groups in the same order,
+// packed_off = g * idx_off; and row / slot counts that fit the int32
+// coordinates of the gather loads.
+bool dense_plan_ok(const rolesub_shape *s, const PlanView &pv)
+{
+    const rolesub_plan &P = *pv.hdr;
+    const int64_t g = (int64_t)s->num_heads * s->head_dim / 16;
+    int64_t r = 0, ix = 0;
+    for (int i = 0; i < P.num_segments; ++i) {
+        const rolesub_segment &sg = pv.segs[i];
+        if (sg.token_row != r || sg.idx_off != ix || sg.packed_off != g * ix) return false;
+        r += sg.n_tokens;
+        ix += (int64_t)sg.n_tokens * sg.k;
+    }
+    const int64_t L = s->num_layers;
+    return r == P.rows_per_layer && ix == P.idx_bytes_per_layer && P.packed_elems_per_layer == g * ix &&
+           L * P.rows_per_layer < ((int64_t)1 << 31) && L * ix < ((int64_t)1 << 31);
+}
+
+// Upper bound on the 128-pair tiles of any chunk: ceil(pairs / 128) plus one
+// partial tile per group.
+int dense_tiles_per_chunk(const PlanView &pv, int chunks)
+{
+    const rolesub_plan &P = *pv.hdr;
+    int best = 0;
+    int i = 0;
+    for (int c = 0; c < chunks; ++c) {
+        const int64_t c0 = (int64_t)c * rs::kDenseChunk, c1 = std::min(P.rows_per_layer, c0 + rs::kDenseChunk);
+        int64_t pairs = 0;
+        while (i < P.num_segments && pv.segs[i].token_row + pv.segs[i].n_tokens <= c0) ++i;
+        for (int j = i; j < P.num_segments && pv.segs[j].token_row < c1; ++j) {
+            const rolesub_segment &sg = pv.segs[j];
+            const int64_t a = std::max(c0, sg.token_row), b = std::min(c1, sg.token_row + sg.n_tokens);
+            if (b > a) pairs += (b - a) * sg.k;
+        }
+        best = std::max(best, (int)((pairs + 127) / 128) + 16);
+    }
+    return best;
 }
 
 bool budget_supported(const rolesub_shape *s, const PlanView &pv)
@@ -606,7 +665,8 @@ rolesub_status rolesub_compress_dense(const rolesub_shape *shape, const void *pl
     if (P.packed_elems_per_layer > 0 && (!packed_v || !aligned16(packed_v))) return ROLESUB_EINVAL;
     if (P.idx_bytes_per_layer > 0 && (!idx || !aligned16(idx))) return ROLESUB_EINVAL;
     if (!isfinite(alpha_role) || !isfinite(alpha_lang)) return ROLESUB_EINVAL;
-    if (!dense_supported(shape) || !rs::router_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    if (!dense_supported(shape) || !rs::router_supported(shape) || !dense_plan_ok(shape, pv))
+        return ROLESUB_EUNSUPPORTED;
     const WsSizes w = ws_sizes(shape, pv.hdr);
     if (ws_bytes < w.total + dense_extra_bytes(shape, pv.hdr)) return ROLESUB_EINVAL;
     rs::CompressArgs a{};
@@ -627,20 +687,36 @@ rolesub_status rolesub_compress_dense(const rolesub_shape *shape, const void *pl
     a.packed = packed_v;
     a.idx = idx;
     a.stream = (cudaStream_t)stream;
-    const int L = shape->num_layers, d = shape->num_heads * shape->head_dim;
-    const int64_t rows = P.rows_per_layer;
-    void *Z = static_cast<char *>(workspace) + w.total;
+    const int L = shape->num_layers, d = shape->num_heads * shape->head_dim, g = d / 16;
+    const DenseWs dw = dense_ws(shape, pv.hdr);
+    char *xb = static_cast<char *>(workspace) + w.total;
+    int2 *pairs = reinterpret_cast<int2 *>(xb + dw.vt + dw.perm + dw.ident);
+    int32_t *meta = reinterpret_cast<int32_t *>(xb + dw.vt + dw.perm + dw.ident + dw.pairs);
     cudaError_t e = rs::launch_router(a);
     if (e != cudaSuccess) return ROLESUB_ECUDA;
     // indices 0..S-1 of k = S rows (the records it also writes are not used)
     e = rs::launch_row_store(pv, L, idx, P.idx_bytes_per_layer, true, reinterpret_cast<uint4 *>(a.ws.row_store),
                              a.ws.status, a.stream);
     if (e != cudaSuccess) return ROLESUB_ECUDA;
-    // Z = V R (z = R^T v for every row, all d dims)
-    e = rs::launch_gemm_tc(true, L, (int)rows, d, d, v, rows * d, R_dense, (int64_t)d * d, Z, rows * d, a.ws.status,
-                           a.stream);
+    if (P.idx_bytes_per_layer == 0) return ROLESUB_OK;
+    // the kept (row, group) pairs per chunk and group, then z_s = R_s^T v of
+    // each pair straight to its packed slot
+    const int chunks = dense_chunks(pv.hdr);
+    e = rs::launch_dense_pairs(pv, L, g, idx, pairs, meta, chunks, a.ws.status, a.stream);
     if (e != cudaSuccess) return ROLESUB_ECUDA;
-    return from_cuda(rs::launch_pack_dense(a, Z));
+    rs::DenseCompressGemm gp{};
+    gp.rows = P.rows_per_layer;
+    gp.d = d;
+    gp.g = g;
+    gp.nt = std::min(g, 256);
+    gp.chunks = chunks;
+    gp.pairs = pairs;
+    gp.pairs_per_layer = P.idx_bytes_per_layer;
+    gp.meta = meta;
+    gp.packed = static_cast<__nv_bfloat16 *>(packed_v);
+    gp.packed_per_layer = P.packed_elems_per_layer;
+    gp.status = a.ws.status;
+    return from_cuda(rs::launch_dense_compress_gemm(gp, v, R_dense, L, dense_tiles_per_chunk(pv, chunks), a.stream));
 }
 
 rolesub_status rolesub_attend_dense(const rolesub_shape *shape, const void *plan_host, const void *plan_dev,
@@ -664,13 +740,15 @@ rolesub_status rolesub_attend_dense(const rolesub_shape *shape, const void *plan
     for (int64_t x : strides)
         if (x < 0 || x % 8 != 0) return ROLESUB_EINVAL;
     if (!isfinite(softmax_scale) || softmax_scale < 0.f) return ROLESUB_EINVAL;
-    if (!dense_supported(shape)) return ROLESUB_EUNSUPPORTED;
+    if (!dense_supported(shape) || !dense_plan_ok(shape, pv)) return ROLESUB_EUNSUPPORTED;
     const WsSizes w = ws_sizes(shape, pv.hdr);
     if (ws_bytes < w.total + dense_extra_bytes(shape, pv.hdr)) return ROLESUB_EINVAL;
-    const int L = shape->num_layers, d = shape->num_heads * shape->head_dim;
+    const int L = shape->num_layers, d = shape->num_heads * shape->head_dim, g = d / 16;
     const int64_t rows = P.rows_per_layer;
-    const size_t vals = align_up(2 * (size_t)L * (size_t)rows * d, kAlign);
-    char *Zm = static_cast<char *>(workspace) + w.total, *Vt = Zm + vals, *Rid = Vt + vals;
+    const DenseWs dw = dense_ws(shape, pv.hdr);
+    char *Vt = static_cast<char *>(workspace) + w.total;
+    int32_t *perm = reinterpret_cast<int32_t *>(Vt + dw.vt);
+    char *Rid = Vt + dw.vt + dw.perm;
     rs::AttendArgs a;
     a.shape = shape;
     a.plan = pv;
@@ -688,13 +766,31 @@ rolesub_status rolesub_attend_dense(const rolesub_shape *shape, const void *plan
     a.scale = softmax_scale;
     a.o = o;
     a.stream = (cudaStream_t)stream;
-    // M z of every row, then v~ = (M z) R^T = R M z back in the original space
-    cudaError_t e = rs::launch_unpack_dense(a, Zm);
+    // rows bucketed by kept-group set (and the attention's records pointing
+    // at their sorted positions), then v~ = R M z over the kept groups only
+    cudaError_t e = rs::launch_dense_sort(pv, L, d, shape->head_dim, idx, perm,
+                                          reinterpret_cast<uint4 *>(a.ws.row_store), a.ws.status, a.stream);
     if (e != cudaSuccess) return ROLESUB_ECUDA;
-    e = rs::launch_gemm_tc(false, L, (int)rows, d, d, Zm, rows * d, R_dense, (int64_t)d * d, Vt, rows * d,
-                           a.ws.status, a.stream);
+    if (P.idx_bytes_per_layer > 0) {
+        rs::DenseAttendGemm gp{};
+        gp.rows = rows;
+        gp.d = d;
+        gp.g = g;
+        gp.G = shape->num_groups;
+        gp.segs = pv.segs_dev;
+        gp.row_seg = pv.row_seg_dev;
+        gp.idx = idx;
+        gp.idx_per_layer = P.idx_bytes_per_layer;
+        gp.slots_per_layer = P.idx_bytes_per_layer;
+        gp.perm = perm;
+        gp.vt = reinterpret_cast<__nv_bfloat16 *>(Vt);
+        gp.status = a.ws.status;
+        e = rs::launch_dense_attend_gemm(gp, packed_v, R_dense, L, a.stream);
+    } else if (rows > 0) {
+        e = cudaMemsetAsync(Vt, 0, 2 * (size_t)L * rows * d, a.stream);   // nothing kept: v~ = 0
+    }
     if (e != cudaSuccess) return ROLESUB_ECUDA;
-    e = rs::launch_dense_attend_prep(a, Rid);
+    e = rs::launch_dense_identity(L, shape->num_heads, shape->head_dim, Rid, a.stream);
     if (e != cudaSuccess) return ROLESUB_ECUDA;
     // attention over v~ as plain per-head values (every group kept, R_h = I)
     a.packed = Vt;

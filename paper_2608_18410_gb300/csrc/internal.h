@@ -2,6 +2,7 @@
 // kernel translation units. Not part of the public ABI.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -118,16 +119,49 @@ cudaError_t launch_row_store_budget(const PlanView &pv, int L, const uint8_t *id
 cudaError_t launch_select_tokens(int64_t groups, int n, int k, const float *scores, const void *x, int64_t row_bytes,
                                  int32_t *keep_idx, void *x_keep, cudaStream_t stream);
 
-// Dense rotation (one d x d R per layer): C = A B^T or A B on the tensor core
-// (gemm_tc.cu); packing of the kept d/S-wide groups of Z, the scatter of
-// M z back to [rows][d], and the attention records / identity rotations that
-// let the attention kernel read v~ = R M z as plain values (dense.cu).
-cudaError_t launch_gemm_tc(bool b_mn_major, int L, int M, int N, int K, const void *A, int64_t a_layer_stride,
-                           const void *B, int64_t b_layer_stride, void *C, int64_t c_layer_stride, int32_t *status,
-                           cudaStream_t stream);
-cudaError_t launch_pack_dense(const CompressArgs &a, const void *Z);
-cudaError_t launch_unpack_dense(const AttendArgs &a, void *Zm);
-cudaError_t launch_dense_attend_prep(const AttendArgs &a, void *R_identity);
+// Dense rotation (one d x d R per layer, S = 16 groups of g = d / S rotated
+// dims). Compress: the kept (row, group) pairs of every 4096-row chunk,
+// listed per group (dense.cu), then z of each pair on the tensor core,
+// written to its packed slot (gemm_tc.cu). Attend: the rows of every layer
+// bucketed by kept-group set, with attention records pointing at the sorted
+// rows of v~ (dense.cu), then v~ = R M z on the tensor core over the kept
+// groups only, read from the packed cache (gemm_tc.cu).
+constexpr int kDenseChunk = 4096;       // rows per pair-list chunk
+constexpr int kDenseMetaStride = 32;    // int32 per (layer, chunk): 16 counts, pair base
+struct DenseCompressGemm {
+    int64_t rows;                // cache rows per layer
+    int d, g, nt;                // d = H d_h; g = d / 16; N tile min(g, 256)
+    int chunks;                  // ceil(rows / kDenseChunk)
+    const int2 *pairs;           // [L][pairs_per_layer] {row, packed slot}
+    int64_t pairs_per_layer;     // = idx bytes per layer
+    const int32_t *meta;         // [L][chunks][kDenseMetaStride]
+    __nv_bfloat16 *packed;
+    int64_t packed_per_layer;
+    int32_t *status;
+};
+struct DenseAttendGemm {
+    int64_t rows;
+    int d, g, G;
+    const rolesub_segment *segs;  // device plan
+    const int32_t *row_seg;
+    const uint8_t *idx;
+    int64_t idx_per_layer;
+    int64_t slots_per_layer;      // packed elements per layer / g
+    const int32_t *perm;          // [L][rows]: sorted position -> row
+    __nv_bfloat16 *vt;            // [L][rows][d]: v~ in sorted row order
+    int32_t *status;
+};
+cudaError_t launch_dense_pairs(const PlanView &pv, int L, int g, const uint8_t *idx, int2 *pairs, int32_t *meta,
+                               int chunks, int32_t *status, cudaStream_t stream);
+cudaError_t launch_dense_compress_gemm(const DenseCompressGemm &p, const void *v, const void *R, int L,
+                                       int tiles_per_chunk, cudaStream_t stream);
+cudaError_t launch_dense_sort(const PlanView &pv, int L, int d, int dh, const uint8_t *idx, int32_t *perm,
+                              uint4 *recs, int32_t *status, cudaStream_t stream);
+cudaError_t launch_dense_attend_gemm(const DenseAttendGemm &p, const void *packed, const void *R, int L,
+                                     cudaStream_t stream);
+// Identity R_h of every (layer, head), so that the attention kernel reads
+// v~ as plain per-head values.
+cudaError_t launch_dense_identity(int L, int H, int dh, void *R_identity, cudaStream_t stream);
 
 // Adds n to the process-wide launch counter (rolesub_launch_count).
 void count_launches(int n);

@@ -461,7 +461,7 @@ class RoleSub:
     def compress_dense(self, h, v, R_dense, W_re, b_re, W1, b1, W2, b2, alpha_role=0.1, alpha_lang=0.1,
                        packed=None, idx=None, stream=None):
         """Dense-rotation compress; the first call allocates its larger
-        workspace (two [L][rows][d] bf16 buffers)."""
+        workspace (one [L][rows][d] bf16 buffer and the pair lists)."""
         if packed is None or idx is None:
             packed, idx = self.new_outputs()
         ws = self._dense_workspace()

@@ -251,7 +251,7 @@ def test_select_tokens_rejects_bad_arguments_before_any_launch(rsm):
 
 
 def test_dense_calls_reject_bad_arguments_before_any_launch(rsm):
-    shape = rsm.make_shape(1, 4, 128, 16, 8, 32, "bf16")
+    shape = rsm.make_shape(1, 8, 128, 16, 8, 32, "bf16")   # d = 1024, g = 64
     plan = rsm.Plan(shape, [[3, 2, 0, 0]], [[4, 16, 16, 16]], [1])
     L = rsm.lib()
     fake = 1 << 20
@@ -266,14 +266,21 @@ def test_dense_calls_reject_bad_arguments_before_any_launch(rsm):
     a = list(args)
     a[17] = big - 256                   # workspace without the dense buffers
     assert L.rolesub_compress_dense(*a) == 1
-    odd = rsm.make_shape(1, 3, 128, 16, 8, 32, "bf16")     # d = 384: not a multiple of 256
-    po = rsm.Plan(odd, [[3, 2, 0, 0]], [[4, 16, 16, 16]], [1])
-    a = list(args)
-    a[0], a[1] = ctypes.byref(odd), po.host_ptr
-    assert L.rolesub_compress_dense(*a) == 2
-    at = [ctypes.byref(shape), plan.host_ptr, fake, fake, 0, 512, 128, fake, 0, 512, 128, fake, fake, fake,
+    for H in (3, 4, 6):
+        # d = 384 (not a multiple of 256), g = 32 (less than a 64-wide K
+        # block), g = 48: unsupported group geometry
+        odd = rsm.make_shape(1, H, 128, 16, 8, 32, "bf16")
+        po = rsm.Plan(odd, [[3, 2, 0, 0]], [[4, 16, 16, 16]], [1])
+        a = list(args)
+        a[0], a[1] = ctypes.byref(odd), po.host_ptr
+        a[17] = po.dense_workspace_size()
+        assert L.rolesub_compress_dense(*a) == 2, H
+    at = [ctypes.byref(shape), plan.host_ptr, fake, fake, 0, 1024, 128, fake, 0, 1024, 128, fake, fake, fake,
           0.0, fake, fake, big, None]
     at[13] = None                       # R_dense
+    assert L.rolesub_attend_dense(*at) == 1
+    at[13] = fake
+    at[17] = big - 256
     assert L.rolesub_attend_dense(*at) == 1
 
 

@@ -96,11 +96,28 @@ def _run(wl, pairs):
 
 
 def test_dense_ragged_episodes():
+    # g = 64: one K block per group; k from 0 to 16, empty kinds, a
+    # single-token segment, more than 128 pairs of one group
     E = synth.Episode
     eps = [E(130, 20, 64, 4, 16), E(9, 3, 5, 2, 1), E(0, 6, 3, 3, 3), E(33, 0, 70, 16, 0),
            E(40, 9, 9, 15, 1, n_prop=3, n_act=8)]
-    wl = synth.Workload("dense_edge", "bf16", L=2, H=4, dh=128, G=16, C=8, F=32, episodes=tuple(eps), seed=41)
+    wl = synth.Workload("dense_edge", "bf16", L=2, H=8, dh=128, G=16, C=8, F=32, episodes=tuple(eps), seed=41)
     _run(wl, [(l, e) for l in range(2) for e in range(len(eps))])
+
+
+def test_dense_g128_several_chunks():
+    # g = 128 (N tile 128 in the z GEMM, two K blocks per group) and more
+    # than 4096 rows per layer: pair lists of two chunks, a ragged last
+    # chunk, many 128-row tiles of v~; sampled episodes checked
+    E = synth.Episode
+    rng = np.random.default_rng(7)
+    eps = [E(int(rng.integers(120, 300)), int(rng.integers(8, 40)), 4, int(rng.choice([2, 4, 8])),
+             int(rng.choice([1, 4, 16]))) for _ in range(22)]
+    eps[3] = E(200, 10, 4, 0, 0)        # nothing kept
+    wl = synth.Workload("dense_chunks", "bf16", L=1, H=16, dh=128, G=16, C=8, F=32, episodes=tuple(eps),
+                        seed=43)
+    assert sum(e.n_cache for e in eps) > 4096
+    _run(wl, [(0, e) for e in (0, 3, 11, 21)])
 
 
 def test_dense_oft_layer():
