@@ -21,18 +21,17 @@
 // zeroed with tcgen05.st first.
 //
 // One CTA per tile, 192 threads: warps 0-3 set the tile up, gather A with
-// 16-byte cp.async into the 128-byte-swizzled K-major layout (thread t: the
-// 16-byte column t % 8 of rows t / 8 + 16 i; a TMA tile::gather4 per four
-// rows ran at about a quarter of the MMA rate), and run the epilogue (a TMEM
-// lane and a tile row per thread); warp 4 loads B by TMA; warp 5 issues the
-// MMAs. K runs in 64-wide blocks through a 2-stage ring of 48 KB stages; a
-// gatherer arrives on a stage's barrier once its copies of that stage have
-// landed (one stage later, after a proxy fence). Two CTAs share an SM (about
-// 106 KB of shared memory and 256 TMEM columns each), so that one CTA's
-// set-up and epilogue overlap the other's main loop: measured on the c4
-// cache, 4 stages with one CTA per SM were 10 % slower, 3 stages 40-60 %. The
-// epilogue stages the bf16 tile in the drained ring and stores one tile row
-// (up to 512 bytes) per warp instruction.
+// 16-byte cp.async into the 128-byte-swizzled K-major layout (a TMA
+// tile::gather4 per four rows ran at about a quarter of the MMA rate), and
+// run the epilogue (a TMEM lane and a tile row per thread); warp 4 loads B by
+// TMA; warp 5 issues the MMAs. K runs in 64-wide blocks through a 2-stage
+// ring of 48 KB stages. The gatherers form one team per stage (warps 0-1 the
+// even K blocks, warps 2-3 the odd ones); a team waits for its own copies,
+// fences them to the tensor core's proxy and arrives, so both stages are in
+// flight at once. Two CTAs share an SM (about 106 KB of shared memory and 256
+// TMEM columns each), so that one CTA's set-up and epilogue overlap the
+// other's main loop. The epilogue stages the bf16 tile in the drained ring
+// and stores one tile row (up to 512 bytes) per warp instruction.
 #include <cuda.h>
 
 #include "common.cuh"
@@ -55,11 +54,13 @@ constexpr uint32_t kGTileB = kBN * kBK * 2;          // 32 KB
 constexpr uint32_t kGStage = kGTileA + kGTileB;      // 48 KB
 constexpr uint32_t kGOffBar = kGStages * kGStage;    // 192 KB
 constexpr uint32_t kGOffTab = kGOffBar + 128;
-constexpr int kLag = 1;                              // stages between a gather and its arrival
-constexpr uint32_t kFullCount = 4 * 32 + 1;          // gatherer threads + the B loader
-// a stage is refilled only after its previous round was consumed, which
-// needs that round signalled: at most kGStages - 1 stages may be unsignalled
-static_assert(kLag >= 1 && kLag < kGStages, "gather lag below the ring depth");
+// The gatherers are warps 0-3 as kGStages teams of 128 / kGStages threads;
+// team q fills the stages kb with kb % kGStages == q, waits for its own
+// copies and arrives at once, so every stage of the ring is in flight.
+constexpr int kTeam = 128 / kGStages;                 // threads per gather team
+constexpr int kRowsPerThread = kBM * 8 / kTeam;       // 16-byte chunks per thread and stage
+constexpr uint32_t kFullCount = kTeam + 1;            // the team's threads + the B loader
+static_assert(kRowsPerThread * kTeam == kBM * 8, "a team covers the A tile");
 // attend: slot table [16][128] int32, the lane masks [16][4] uint32, kept
 // groups per row [128] uint32; compress: A row per tile row [128] int32,
 // then packed offsets [128] int64
@@ -69,22 +70,13 @@ constexpr uint32_t kGPitch = kBN * 2 + 16;           // staged C row: 512 B + 16
 static_assert(kBM * kGPitch <= kGOffBar, "C staging fits the ring");
 static_assert(kBM * 4 + kBM * 8 <= kGTabBytes, "compress tables fit");
 
-// This thread's part of a stage's A gather is complete: its copies of stage
-// `kb - kLag` have landed (program order of the cp.async groups); they are
-// made visible to the tensor core's proxy, then the stage barrier arrives.
-__device__ __forceinline__ void gather_signal(uint32_t bar_full, int kb)
-{
-    cp_async_wait_group<kLag>();
-    fence_async_smem();
-    mbar_arrive(bar_full + 8 * ((kb - kLag) % kGStages));
-}
-
-// After the last stage: every copy landed, arrivals for the last kLag stages.
-__device__ __forceinline__ void gather_finish(uint32_t bar_full, int issued)
+// This thread's copies of the stage have landed: made visible to the tensor
+// core's proxy, then the stage barrier arrives.
+__device__ __forceinline__ void gather_done(uint32_t full)
 {
     cp_async_wait_group<0>();
     fence_async_smem();
-    for (int kb = max(0, issued - kLag); kb < issued; ++kb) mbar_arrive(bar_full + 8 * (kb % kGStages));
+    mbar_arrive(full);
 }
 
 // D[tmem] += A . B^T on the lanes whose bit in dis[] is clear (bit i of
@@ -186,30 +178,28 @@ k_dense_compress_tc(const __grid_constant__ CUtensorMap tm_r, const bf16 *__rest
 
     if (warp < 4) {
         // ------------------------------------- A gather, then the epilogue
-        const int cc = tid & 7, rq = tid >> 3;
-        const bf16 *src[8];
-        uint32_t doff[8], valid = 0;
+        // thread: team q, the 16-byte column cc of rows rq + 8 i
+        const int q = tid / kTeam, tt = tid % kTeam, cc = tt & 7, rq = tt >> 3;
+        const bf16 *src[kRowsPerThread];
+        uint32_t doff[kRowsPerThread], valid = 0;
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const int row = rq + 16 * i;
+        for (int i = 0; i < kRowsPerThread; ++i) {
+            const int row = rq + (kTeam / 8) * i;
             src[i] = v + (int64_t)arow[row] * p.d + 8 * cc;
             doff[i] = (uint32_t)row * 128u + ((uint32_t)(cc ^ (row & 7)) << 4);
             if (row < nvalid) valid |= 1u << i;
         }
-        int kb = 0;
-        for (; kb < nkb; ++kb) {
-            const int st_i = kb % kGStages;
+        for (int kb = q; kb < nkb; kb += kGStages) {
             if (kb >= kGStages &&
-                !mbar_wait(bar_empty + 8 * st_i, ((kb / kGStages) - 1) & 1, p.status, &abort_flag, 95))
+                !mbar_wait(bar_empty + 8 * q, ((kb / kGStages) - 1) & 1, p.status, &abort_flag, 95))
                 break;
-            const uint32_t st = sb + kGStage * st_i;
+            const uint32_t st = sb + kGStage * q;
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
+            for (int i = 0; i < kRowsPerThread; ++i)
                 if ((valid >> i) & 1u) cp_async16(st + doff[i], src[i] + kBK * kb);
             cp_async_commit();
-            if (kb >= kLag) gather_signal(bar_full, kb);
+            gather_done(bar_full + 8 * q);
         }
-        gather_finish(bar_full, kb);
 
         const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
         const bool ok = mbar_wait(bar_acc, 0, p.status, &abort_flag, 97);
@@ -357,40 +347,45 @@ k_dense_attend_tc(const __grid_constant__ CUtensorMap tm_r, const bf16 *__restri
 
     if (warp < 4) {
         // ------------------------------------- A gather, then the epilogue
-        const int cc = tid & 7, rq = tid >> 3;
-        uint32_t kp[8], doff[8];
+        // thread: team q, the 16-byte column cc of rows rq + 8 i
+        const int q = tid / kTeam, tt = tid % kTeam, cc = tt & 7, rq = tt >> 3;
+        uint32_t kp[kRowsPerThread], doff[kRowsPerThread];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            const int row = rq + 16 * i;
+        for (int i = 0; i < kRowsPerThread; ++i) {
+            const int row = rq + (kTeam / 8) * i;
             kp[i] = keeps[row];
             doff[i] = (uint32_t)row * 128u + ((uint32_t)(cc ^ (row & 7)) << 4);
         }
         uint32_t rest = un;
-        int s = -1, sub = kpg, kb = 0;
-        const bf16 *src[8];
-        for (; kb < nkb; ++kb) {
+        int s = -1, sub = kpg;
+        uint32_t on = 0;                  // rows of this thread that kept s
+        const bf16 *src[kRowsPerThread];  // their slots of group s
+        for (int kb = 0; kb < nkb; ++kb) {
             if (sub == kpg) {
                 s = __ffs(rest) - 1;
                 rest &= rest - 1;
                 sub = 0;
+                on = 0;
 #pragma unroll
-                for (int i = 0; i < 8; ++i)
-                    src[i] = packed + (int64_t)slot[s * kBM + rq + 16 * i] * g + 8 * cc;
+                for (int i = 0; i < kRowsPerThread; ++i) {
+                    on |= ((kp[i] >> s) & 1u) << i;
+                    src[i] = packed + (int64_t)slot[s * kBM + rq + (kTeam / 8) * i] * g + 8 * cc;
+                }
             }
-            const int st_i = kb % kGStages;
-            if (kb >= kGStages &&
-                !mbar_wait(bar_empty + 8 * st_i, ((kb / kGStages) - 1) & 1, p.status, &abort_flag, 99))
-                break;
-            const uint32_t st = sb + kGStage * st_i;
-            // rows that did not keep s load nothing: their lanes are masked
+            if (kb % kGStages == q) {
+                if (kb >= kGStages &&
+                    !mbar_wait(bar_empty + 8 * q, ((kb / kGStages) - 1) & 1, p.status, &abort_flag, 99))
+                    break;
+                const uint32_t st = sb + kGStage * q;
+                // rows that did not keep s load nothing: their lanes are masked
 #pragma unroll
-            for (int i = 0; i < 8; ++i)
-                if ((kp[i] >> s) & 1u) cp_async16(st + doff[i], src[i] + kBK * sub);
-            cp_async_commit();
-            if (kb >= kLag) gather_signal(bar_full, kb);
+                for (int i = 0; i < kRowsPerThread; ++i)
+                    if ((on >> i) & 1u) cp_async16(st + doff[i], src[i] + kBK * sub);
+                cp_async_commit();
+                gather_done(bar_full + 8 * q);
+            }
             ++sub;
         }
-        gather_finish(bar_full, kb);
 
         const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
         const bool ok = mbar_wait(bar_acc, 0, p.status, &abort_flag, 100);
