@@ -712,11 +712,16 @@ def run_ours(args):
     cab = compress_additive_bytes(wl, C_ADD)
     comp_add = {"ms": add_ms, "role_dim": C_ADD, "algorithmic_bytes": cab, "GB/s": cab / (add_ms / 1e3) / 1e9,
                 "frac": cab / (add_ms / 1e3) / 1e9 / peaks["hbm_gbs"]}
-    gemm_flop = 2.0 * wl.rows * wl.d * wl.d * wl.L     # one d x d rotation of every cache row, all layers
+    # only kept groups are rotated: z_s = R_s^T v (compress) and v~ = sum over
+    # kept s of R_s z_s (attend), 2 g d flop per kept (row, group) pair each
+    kept_pairs = int((wl.n_tok_array().astype(np.int64) * wl.k_array()).sum()) * wl.L
+    kept_flop = 2.0 * (wl.d // wl.G) * wl.d * kept_pairs
     dense = {"compress_ms": den_c_ms, "attend_ms": den_a_ms,
-             "rotation_gemm_tflop": gemm_flop / 1e12,
-             "compress_tflops_rotation_only": gemm_flop / (den_c_ms / 1e3) / 1e12,
-             "attend_tflops_rotation_only": gemm_flop / (den_a_ms / 1e3) / 1e12,
+             "kept_pairs": kept_pairs,
+             "rotation_tflop_kept": kept_flop / 1e12,
+             "compress_tflops_kept": kept_flop / (den_c_ms / 1e3) / 1e12,
+             "attend_tflops_kept": kept_flop / (den_a_ms / 1e3) / 1e12,
+             "all_groups_tflop": 2.0 * wl.rows * wl.d * wl.d * wl.L / 1e12,
              "query_tokens_per_s_per_layer": qtok / ((den_c_ms + den_a_ms) / 1e3),
              "r": "one d x d orthonormal R per layer (kron of two 64 x 64 Haar factors)"}
     latency = {"workload": wl1.name, "l2": "flushed before each step", "eager_ms": lat_eager,

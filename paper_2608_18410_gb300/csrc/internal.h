@@ -105,6 +105,8 @@ cudaError_t launch_attend(const AttendArgs &a);
 // Routed attention on tcgen05/TMA (bf16, d_h = 128, S = 16).
 bool attend_tc_supported(const rolesub_shape *s);
 cudaError_t launch_attend_tc(const AttendArgs &a);
+// The same for a budget cache (a.k_tok set); launch_attend_tc dispatches.
+cudaError_t launch_attend_tc_budget(const AttendArgs &a);
 
 // Per-token budgets (Sec. 3.5): from the scores and priorities of score
 // mode, the counts K_i of every routed segment, the kept groups at prefix
