@@ -134,13 +134,19 @@ def load_peaks():
 def load_traffic(kernel, workload):
     """DRAM bytes per launch from a committed ncu summary, if it is current.
 
-    profiles/traffic.txt lines: kernel workload source_sha256 dram_bytes
+    profiles/traffic.txt lines: kernel workload source_sha256[:16] dram_bytes,
+    the hash taken over csrc/<kernel>.cuh when it exists, else <kernel>.cu
     """
     import hashlib
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
-    src = os.path.join(ROOT, "paper_2608_18410_gb300", "csrc", kernel + ".cu")
+    # the file that holds the kernel's code (the attention kernel is a header
+    # shared by its fixed-k and budget translation units)
+    csrc = os.path.join(ROOT, "paper_2608_18410_gb300", "csrc")
+    src = os.path.join(csrc, kernel + ".cuh")
+    if not os.path.exists(src):
+        src = os.path.join(csrc, kernel + ".cu")
     if not os.path.exists(src):
         return None
     sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]

@@ -52,7 +52,7 @@ constexpr int kMaxGroups = 16;
 constexpr uint32_t kGTileA = kBM * kBK * 2;          // 16 KB
 constexpr uint32_t kGTileB = kBN * kBK * 2;          // 32 KB
 constexpr uint32_t kGStage = kGTileA + kGTileB;      // 48 KB
-constexpr uint32_t kGOffBar = kGStages * kGStage;    // 192 KB
+constexpr uint32_t kGOffBar = kGStages * kGStage;    // 96 KB
 constexpr uint32_t kGOffTab = kGOffBar + 128;
 // The gatherers are warps 0-3 as kGStages teams of 128 / kGStages threads;
 // team q fills the stages kb with kb % kGStages == q, waits for its own
