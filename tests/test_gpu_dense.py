@@ -123,3 +123,15 @@ def test_dense_g128_several_chunks():
 def test_dense_oft_layer():
     wl = synth.c1()
     _run(wl, [(0, 0)])
+
+
+@pytest.mark.slow
+def test_dense_c4_full_size_sampled():
+    # the bench's workload and launch configuration: 64 ragged episodes x 32
+    # layers, d = 4096, g = 256 (three pair-list chunks and 91 row tiles of
+    # v~ per layer); sampled (layer, episode) pairs, the largest and the
+    # smallest episode included
+    wl = synth.c4()
+    sizes = [ep.n_cache for ep in wl.episodes]
+    e_big, e_small = int(np.argmax(sizes)), int(np.argmin(sizes))
+    _run(wl, [(0, e_big), (31, e_small), (17, 5), (5, 40)])
