@@ -183,7 +183,7 @@ template <bool kBudget>
 __global__ void __launch_bounds__(kBudget ? kThreadsBudget : kThreads, 1)
 k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_k,
             const __grid_constant__ CUtensorMap tm_r, const bf16 *__restrict__ packed,
-            int64_t packed_per_layer, const uint4 *__restrict__ rec, int64_t rows,
+            int64_t packed_per_layer, const uint4 *rec, int64_t rows,
             const rolesub_episode *__restrict__ eps, int E, int H, int qtiles, int64_t u0, int64_t u1, int64_t q_rows,
             float scale_log2, bf16 *__restrict__ o, int32_t *status)
 {
@@ -440,7 +440,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             mnext = make_uint4(0, 0, 0, 0);
             if (ahead.k < nu) {
                 const int r = ahead.c * kChunk + jl;
-                if (r < ahead.t.nc) mnext = __ldg(rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
+                if (r < ahead.t.nc) mnext = ld_dep(rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
             }
             for (int i = 0; i < kGath; ++i) it_next(sp, ahead, nu);
         };
@@ -499,7 +499,7 @@ k_attend_tc(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CU
             mnext = make_uint4(0, 0, 0, 0);
             if (ahead.k < nu) {
                 const int r = ahead.c * kChunk + jl;
-                if (r < ahead.t.nc) mnext = __ldg(rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
+                if (r < ahead.t.nc) mnext = ld_dep(rec + (int64_t)ahead.t.l * rows + ahead.t.krow + r);
             }
             it_next(sp, ahead, nu);
             it_next(sp, ahead, nu);

@@ -80,7 +80,7 @@ __device__ __forceinline__ uint4 record(uint64_t gid, int64_t base8, int k, int6
 
 // Shared memory: pri [n] order keys | rem [n] u32 | pre [n] i32 | kk [n] u8
 __global__ void __launch_bounds__(kBT)
-k_budget_select(PlanDev plan, int64_t rows, const float *__restrict__ scores, uint8_t *__restrict__ idx,
+k_budget_select(PlanDev plan, int64_t rows, const float *scores, uint8_t *__restrict__ idx,
                 int64_t idx_per_layer, uint8_t *__restrict__ k_tok, uint4 *__restrict__ recs)
 {
     extern __shared__ __align__(16) uint8_t smb[];
@@ -110,7 +110,7 @@ k_budget_select(PlanDev plan, int64_t rows, const float *__restrict__ scores, ui
         }
         return;
     }
-    for (int i = tid; i < n; i += kBT) pri[i] = order_key(scores[(lrow + row0 + i) * kScoreStride + kG]);
+    for (int i = tid; i < n; i += kBT) pri[i] = order_key(ld_dep(scores + (lrow + row0 + i) * kScoreStride + kG));
     if (tid == 0) {
         int c = 0;   // saturated ranks: the first c whose largest unsaturated share is <= S
         for (; c < n; ++c) {
@@ -169,7 +169,7 @@ k_budget_select(PlanDev plan, int64_t rows, const float *__restrict__ scores, ui
         uint32_t gam[kG];
 #pragma unroll
         for (int q = 0; q < kG / 4; ++q) {
-            const float4 v = sp[q];
+            const float4 v = ld_dep(sp + q);
             gam[4 * q] = order_key(v.x);
             gam[4 * q + 1] = order_key(v.y);
             gam[4 * q + 2] = order_key(v.z);

@@ -23,6 +23,48 @@ constexpr size_t kStatusBytes = 256;
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
+// Loads of what the kernel before this one writes, in a kernel started by
+// launch_pdl. Such a kernel is resident while its predecessor still writes,
+// so that data must not be read through a const __restrict__ pointer or
+// __ldg: the compiler may then take the read-only (non-coherent) path and
+// move the load above pdl_wait(), and the kernel reads stale values (found on
+// the language context, which the bias kernels read as soon as a small
+// pooling grid let them start). These are ordinary global loads in asm
+// volatile, so they stay after the wait.
+__device__ __forceinline__ float ld_dep(const float *p)
+{
+    float v;
+    asm volatile("ld.global.f32 %0, [%1];" : "=f"(v) : "l"(p) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ float4 ld_dep(const float4 *p)
+{
+    float4 v;
+    asm volatile("ld.global.v4.f32 {%0, %1, %2, %3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "l"(p)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ uint4 ld_dep(const uint4 *p)
+{
+    uint4 v;
+    asm volatile("ld.global.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "l"(p)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ uint32_t ld_dep(const uint8_t *p)
+{
+    uint32_t v;
+    asm volatile("ld.global.u8 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
 template <class... P, class... A>
 inline cudaError_t launch_pdl(void (*kern)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
                               A &&...args)

@@ -54,7 +54,7 @@ constexpr uint32_t kIdesc = idesc_bf16(128, 128, true);
 // k = 0 means nothing is stored for the row (or its indices were corrupt).
 // write_identity: also write indices 0..S-1 of k = S rows (compress only).
 __global__ void __launch_bounds__(256)
-k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_per_layer, bool write_identity,
+k_row_store(PlanDev plan, int64_t rows, uint8_t *idx, int64_t idx_per_layer, bool write_identity,
             uint4 *__restrict__ meta, int32_t *status)
 {
     pdl_trigger();
@@ -74,7 +74,7 @@ k_row_store(PlanDev plan, int64_t rows, uint8_t *__restrict__ idx, int64_t idx_p
             for (int s = 0; s < kG; ++s) ix[s] = (uint8_t)s;   // byte stores: no alignment needed
     } else {
         for (int s = 0; s < k; ++s) {
-            const uint32_t g = ix[s];
+            const uint32_t g = ld_dep(ix + s);
             if (g >= kG) {
                 report(status, ROLESUB_EDEVICE, (int)r);
                 kk = 0;
@@ -104,7 +104,7 @@ __device__ __forceinline__ RotItem rot_item(int it, int H, int L, int per, int n
 
 __global__ void __launch_bounds__(kThreads, 1)
 k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CUtensorMap tm_r,
-            const uint4 *__restrict__ meta, int64_t rows, int H, int L, int per, int ntiles, int nitems,
+            const uint4 *meta, int64_t rows, int H, int L, int per, int ntiles, int nitems,
             bf16 *__restrict__ packed, int64_t packed_per_layer, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -219,7 +219,7 @@ k_rotate_tc(const __grid_constant__ CUtensorMap tm_v, const __grid_constant__ CU
             uint4 m = zero4;
             if (ai < nitems) {
                 const int64_t r = (int64_t)(aw.t0 + at) * kRows + tid;
-                if (r < rows) m = __ldg(meta + (int64_t)aw.l * rows + r);
+                if (r < rows) m = ld_dep(meta + (int64_t)aw.l * rows + r);
                 if (++at >= aw.nt) {
                     at = 0;
                     ai += gridDim.x;

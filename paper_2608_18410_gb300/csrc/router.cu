@@ -211,7 +211,7 @@ k_lang_bias(const T *__restrict__ W1, const float *__restrict__ b1, const float 
 constexpr int kGemvEpisodes = 4;
 
 __global__ void __launch_bounds__(256)
-k_lang_bias_gemv(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *__restrict__ ctx,
+k_lang_bias_gemv(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *ctx,
                  int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
 {
     const int l = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -237,7 +237,7 @@ k_lang_bias_gemv(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__
 #pragma unroll
         for (int e = 0; e < kGemvEpisodes; ++e) {
             if (e >= E) break;
-            const float4 x0 = __ldg(c4 + (size_t)e * (d / 4) + 2 * k8), x1 = __ldg(c4 + (size_t)e * (d / 4) + 2 * k8 + 1);
+            const float4 x0 = ld_dep(c4 + (size_t)e * (d / 4) + 2 * k8), x1 = ld_dep(c4 + (size_t)e * (d / 4) + 2 * k8 + 1);
             float a = acc[e];
             a = fmaf(wf[0], x0.x, a);
             a = fmaf(wf[1], x0.y, a);
@@ -293,7 +293,7 @@ __device__ __forceinline__ uint32_t pack2(float a, float b)
 
 template <int kSplit>
 __global__ void __cluster_dims__(kSplit, 1, 1) __launch_bounds__(128)
-k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *__restrict__ ctx,
+k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *ctx,
                 int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
 {
     constexpr int BE = 64, BF = 64, BK = 64;
@@ -318,7 +318,7 @@ k_lang_bias_mma(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ 
 #pragma unroll
         for (int j = 0; j < 8; ++j) {   // ctx: row e, float4 kq of the 64-wide step
             const int idx = tid + 128 * j, e = e0 + (idx >> 4), kq = idx & 15;
-            cr[j] = e < E ? *reinterpret_cast<const float4 *>(cbase + (size_t)e * d + k0 + 4 * kq)
+            cr[j] = e < E ? ld_dep(reinterpret_cast<const float4 *>(cbase + (size_t)e * d + k0 + 4 * kq))
                           : make_float4(0.f, 0.f, 0.f, 0.f);
         }
 #pragma unroll

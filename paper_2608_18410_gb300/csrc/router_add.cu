@@ -39,7 +39,7 @@ typedef __nv_bfloat16 bf16;
 // beta[l][e][s] = alpha_lang * (b_l[l][s] + W_l[l][s] . c[l][e])
 template <class T>
 __global__ void __launch_bounds__(256)
-k_lang_term_add(const T *__restrict__ W_l, const float *__restrict__ b_l, const float *__restrict__ ctx, int E,
+k_lang_term_add(const T *__restrict__ W_l, const float *__restrict__ b_l, const float *ctx, int E,
                 int d, int G, float alpha_lang, float *__restrict__ beta)
 {
     const int l = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -51,7 +51,7 @@ k_lang_term_add(const T *__restrict__ W_l, const float *__restrict__ b_l, const 
     const T *w = W_l + ((size_t)l * G + s) * d;
     const float *c = ctx + ((size_t)l * E + e) * d;
     float acc = 0.f;
-    for (int t = lane; t < d; t += 32) acc = fmaf(to_f(w[t]), c[t], acc);
+    for (int t = lane; t < d; t += 32) acc = fmaf(to_f(w[t]), ld_dep(c + t), acc);
     acc = warp_sum(acc);
     if (lane == 0) beta[((size_t)l * E + e) * G + s] = alpha_lang * (b_l[(size_t)l * G + s] + acc);
 }
@@ -63,7 +63,7 @@ constexpr int kTermEp = 4, kTermMaxG = 16;
 
 template <class T>
 __global__ void __launch_bounds__(256)
-k_lang_term_add4(const T *__restrict__ W_l, const float *__restrict__ b_l, const float *__restrict__ ctx, int E,
+k_lang_term_add4(const T *__restrict__ W_l, const float *__restrict__ b_l, const float *ctx, int E,
                  int d, int G, float alpha_lang, float *__restrict__ beta)
 {
     __shared__ float part[8][kTermEp * kTermMaxG];
@@ -80,7 +80,7 @@ k_lang_term_add4(const T *__restrict__ W_l, const float *__restrict__ b_l, const
     for (int t = threadIdx.x; t < d; t += 256) {
         float cv[kTermEp];
 #pragma unroll
-        for (int i = 0; i < kTermEp; ++i) cv[i] = e0 + i < E ? c[(size_t)i * d + t] : 0.f;
+        for (int i = 0; i < kTermEp; ++i) cv[i] = e0 + i < E ? ld_dep(c + (size_t)i * d + t) : 0.f;
 #pragma unroll
         for (int s = 0; s < kTermMaxG; ++s) {
             if (s < G) {
@@ -192,7 +192,7 @@ __global__ void __launch_bounds__(kTThreads, 2)
 k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_wv,
                 const __grid_constant__ CUtensorMap tm_wre, PlanDev plan, int64_t rows, int d, int C, int E,
                 int nb, int stages, const float *__restrict__ b_v, const float *__restrict__ b_re,
-                const bf16 *__restrict__ W_role, const float *__restrict__ beta, float alpha_role,
+                const bf16 *__restrict__ W_role, const float *beta, float alpha_role,
                 uint8_t *__restrict__ idx, int64_t idx_per_layer, const float *__restrict__ u_pri,
                 float *__restrict__ scores, int32_t *status)
 {
@@ -345,7 +345,7 @@ k_router_add_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant_
             const float *be = beta + ((size_t)l * E + sg.episode) * kTG;
             const float inv = 1.f / z;
 #pragma unroll
-            for (int s = 0; s < kTG; ++s) gam[s] += alpha_role * (acc[s] * inv) + __ldg(be + s);
+            for (int s = 0; s < kTG; ++s) gam[s] += alpha_role * (acc[s] * inv) + ld_dep(be + s);
             if (scores) {
                 // score mode (per-token budgets): gamma and pi to the
                 // workspace, the selection runs once the segment's counts

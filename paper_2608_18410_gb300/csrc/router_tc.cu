@@ -78,7 +78,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CUtensorMap tm_w1,
             const __grid_constant__ CUtensorMap tm_wre, const __grid_constant__ CUtensorMap tm_w2,
             PlanDev plan, int tiles, int L, int64_t rows, int d, int E, int G, const float *__restrict__ b_re,
-            const float *__restrict__ beta, const float *__restrict__ b2, float alpha_role,
+            const float *beta, const float *__restrict__ b2, float alpha_role,
             uint8_t *__restrict__ idx, int64_t idx_per_layer, int32_t *status)
 {
     extern __shared__ uint8_t smem_raw[];
@@ -326,7 +326,7 @@ k_router_tc(const __grid_constant__ CUtensorMap tm_h, const __grid_constant__ CU
                     tmem_wait_ld();
 #pragma unroll
                     for (int cc = 0; cc < 4; ++cc) {
-                        const float4 b0 = __ldg(be + 8 * q + 2 * cc), b1 = __ldg(be + 8 * q + 2 * cc + 1);
+                        const float4 b0 = ld_dep(be + 8 * q + 2 * cc), b1 = ld_dep(be + 8 * q + 2 * cc + 1);
                         const float bb[8] = {b0.x, b0.y, b0.z, b0.w, b1.x, b1.y, b1.z, b1.w};
                         uint32_t hw[4], lw[4];
 #pragma unroll
