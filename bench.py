@@ -34,6 +34,7 @@ sys.path.insert(0, ROOT)
 METRIC = "action-query attend+compress tokens/s per layer; HBM GB/s fraction of peak"
 UNIT = "query tokens/s/layer"
 FLUSH_BYTES = 512 << 20
+E2E_CHUNK = 4   # layers per chunk of the end-to-end pipeline
 
 
 # ---------------------------------------------------------------------------
@@ -664,7 +665,12 @@ def run_ours(args):
     assert code == 0, f"device status {code}"
     del lat_flush, d2, rs2, p2, i2, o2
 
-    # ---- end to end through the public API from pinned host buffers --------
+    # ---- end to end through the public API from pinned host buffers. The
+    # layers go in chunks of E2E_CHUNK: a chunk's activations are copied in
+    # on one stream, compress + attend run on the launching stream, and its
+    # output is copied out on a third, so that copies in, compute and copies
+    # out of neighbouring chunks overlap (the host link bounds the step).
+    # Every step copies all of its inputs in and all of o out. -------------
     act = ("h", "v", "K", "q")
     host = {}
     for k in act:
@@ -676,23 +682,63 @@ def run_ours(args):
     d2h = o_host.numel() * o_host.element_size()
     dv = {k: (d[k].view(torch.int16) if d[k].dtype == torch.bfloat16 else d[k]) for k in act}
     ov = o.view(torch.int16) if o.dtype == torch.bfloat16 else o
+    chunks = [(l0, min(wl.L, l0 + E2E_CHUNK)) for l0 in range(0, wl.L, E2E_CHUNK)]
+    rs_chunk = {}
+    for l0, l1 in chunks:
+        if l1 - l0 not in rs_chunk:
+            rs_chunk[l1 - l0] = rolesub.RoleSub(l1 - l0, wl.H, wl.dh, wl.G, wl.C, wl.F, wl.dtype, wl.n_tok_array(),
+                                                wl.k_array(), wl.n_query_array(), device=dev)
+    outs = [rs_chunk[l1 - l0].new_outputs() for l0, l1 in chunks]   # a chunk's own packed cache and indices
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    ev_in = [torch.cuda.Event() for _ in chunks]
+    ev_done = [torch.cuda.Event() for _ in chunks]
+    ev_out = [torch.cuda.Event() for _ in chunks]
+    e2e_state = {"steps": 0}
 
     def e2e_step():
-        for k in act:
-            dv[k].copy_(host[k], non_blocking=True)
-        compress()
-        attend()
-        o_host.copy_(ov, non_blocking=True)
+        later = e2e_state["steps"] > 0
+        for c, (l0, l1) in enumerate(chunks):
+            if later:
+                s_in.wait_event(ev_done[c])    # the previous step's compute has read this chunk's inputs
+            with torch.cuda.stream(s_in):
+                for k in act:
+                    dv[k][l0:l1].copy_(host[k][l0:l1], non_blocking=True)
+                ev_in[c].record(s_in)
+            stream.wait_event(ev_in[c])
+            if later:
+                stream.wait_event(ev_out[c])   # the previous step's o of this chunk has been copied out
+            r = rs_chunk[l1 - l0]
+            pk, ix = outs[c]
+            r.compress(d["h"][l0:l1], d["v"][l0:l1], d["R"][l0:l1], d["W_re"][l0:l1], d["b_re"][l0:l1],
+                       d["W1"][l0:l1], d["b1"][l0:l1], d["W2"][l0:l1], d["b2"][l0:l1], wl.alpha_role,
+                       wl.alpha_lang, packed=pk, idx=ix, stream=stream)
+            r.attend(d["q"][l0:l1], d["K"][l0:l1], pk, ix, d["R"][l0:l1], o=o[l0:l1], stream=stream)
+            ev_done[c].record(stream)
+            s_out.wait_event(ev_done[c])
+            with torch.cuda.stream(s_out):
+                o_host[l0:l1].copy_(ov[l0:l1], non_blocking=True)
+                ev_out[c].record(s_out)
+        e2e_state["steps"] += 1
 
+    compress()                   # o of the whole-workload calls, to check the chunked steps against
+    attend()
+    o_whole = o.clone()
     for _ in range(2):
         e2e_step()
     torch.cuda.synchronize()
+    e2e_same = bool(torch.equal(o, o_whole))
+    del o_whole
+    for r in rs_chunk.values():
+        code, _ = r.device_status()
+        assert code == 0, f"device status {code}"
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e2e_steps = max(1, min(args.steps, 20))
     barrier(ws)
     e0.record(stream)
+    s_in.wait_stream(stream)     # nothing of the timed steps starts before e0
     for _ in range(e2e_steps):
         e2e_step()
+    stream.wait_stream(s_out)    # e1 after the last output copy
     e1.record(stream)
     torch.cuda.synchronize()
     e2e_ms = max_over_ranks(e0.elapsed_time(e1), ws) / e2e_steps
@@ -749,7 +795,10 @@ def run_ours(args):
             "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
             "config": workload_config(wl, l2_policy(wl)),
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                    "ms_per_step": e2e_ms},
+                    "ms_per_step": e2e_ms,
+                    "pipeline": f"{len(chunks)} chunks of {E2E_CHUNK} layers: copies in, compute, copies out "
+                                "on three streams",
+                    "o_equals_whole_workload_call": e2e_same},
             "gpu_launches": launches,
             "roofline": roof, "compress": comp, "compress_additive": comp_add, "budget": budget,
             "select_tokens": select, "latency_one_layer": latency, "control_step_c2": control, "dense_rotation": dense,
