@@ -135,3 +135,12 @@ def test_dense_c4_full_size_sampled():
     sizes = [ep.n_cache for ep in wl.episodes]
     e_big, e_small = int(np.argmax(sizes)), int(np.argmin(sizes))
     _run(wl, [(0, e_big), (31, e_small), (17, 5), (5, 40)])
+
+
+def test_dense_g512_two_column_tiles():
+    # d = 8192 (64 heads), g = 512: every 128-pair tile of the z GEMM runs as
+    # two 256-column tiles, and a group is eight K blocks of the v~ GEMM
+    E = synth.Episode
+    eps = [E(40, 8, 4, 4, 16), E(7, 3, 3, 2, 1), E(0, 5, 2, 15, 3)]
+    wl = synth.Workload("dense_g512", "bf16", L=1, H=64, dh=128, G=16, C=8, F=32, episodes=tuple(eps), seed=47)
+    _run(wl, [(0, e) for e in range(len(eps))])
