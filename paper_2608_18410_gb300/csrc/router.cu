@@ -207,47 +207,86 @@ k_lang_bias(const T *__restrict__ W1, const float *__restrict__ b1, const float 
 // product is a matrix-vector one, bound by reading W1_c once. A warp per
 // output f walks W1_c's row with 16-byte loads (eight weights per lane and
 // step), multiplies by the episodes' ctx in fp32 and sums the lanes with a
-// butterfly. Needs d % 8 == 0 and C % 8 == 0 (16-byte weight rows).
+// butterfly. The block's 8 warps share the layer's contexts, staged once in
+// shared memory after the wait; each lane's first kGemvBatch weight loads are
+// issued before it (W1 is a caller input), later ones a batch at a time, so
+// that the weight stream keeps loads in flight. Needs d % 8 == 0 and
+// C % 8 == 0 (16-byte weight rows).
 constexpr int kGemvEpisodes = 4;
+constexpr int kGemvBatch = 8;
 
 __global__ void __launch_bounds__(256)
 k_lang_bias_gemv(const __nv_bfloat16 *__restrict__ W1, const float *__restrict__ b1, const float *ctx,
                  int E, int d, int C, int F, float alpha_lang, float *__restrict__ beta)
 {
+    extern __shared__ float4 csm[];   // [E][d / 4]: the layer's contexts
     const int l = blockIdx.y, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int f = blockIdx.x * 8 + warp;
-    pdl_trigger();
-    pdl_wait();   // ctx comes from the pooling kernel
-    if (f >= F) return;
-    const uint4 *w = reinterpret_cast<const uint4 *>(W1 + ((size_t)l * F + f) * (size_t)(2 * d + C) + d + C);
-    const float4 *c4 = reinterpret_cast<const float4 *>(ctx + (size_t)l * E * d);
+    const bool live = f < F;
+    const uint4 *w =
+        reinterpret_cast<const uint4 *>(W1 + ((size_t)l * F + (live ? f : 0)) * (size_t)(2 * d + C) + d + C);
     const int n8 = d / 8;
-    float acc[kGemvEpisodes] = {};
-#pragma unroll 8
-    for (int k8 = lane; k8 < n8; k8 += 32) {
-        const uint4 wv = __ldg(w + k8);
-        const __nv_bfloat162 *wp = reinterpret_cast<const __nv_bfloat162 *>(&wv);
-        float wf[8];
+    pdl_trigger();
+    uint4 wb[kGemvBatch];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float2 t = __bfloat1622float2(wp[i]);
-            wf[2 * i] = t.x;
-            wf[2 * i + 1] = t.y;
+    for (int j = 0; j < kGemvBatch; ++j) {
+        const int k8 = lane + 32 * j;
+        wb[j] = live && k8 < n8 ? __ldg(w + k8) : make_uint4(0, 0, 0, 0);
+    }
+    pdl_wait();   // ctx comes from the pooling kernel
+    {
+        const float4 *c4 = reinterpret_cast<const float4 *>(ctx + (size_t)l * E * d);
+        const int nc = E * (d / 4);
+        for (int i0 = threadIdx.x; i0 < nc; i0 += 4 * 256) {
+            float4 t[4];
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int i = i0 + 256 * q;
+                t[q] = i < nc ? ld_dep(c4 + i) : make_float4(0.f, 0.f, 0.f, 0.f);
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                if (i0 + 256 * q < nc) csm[i0 + 256 * q] = t[q];
+        }
+    }
+    __syncthreads();
+    if (!live) return;
+    float acc[kGemvEpisodes] = {};
+    for (int j0 = 0; 32 * j0 < n8; j0 += kGemvBatch) {
+        if (j0 > 0) {
+#pragma unroll
+            for (int j = 0; j < kGemvBatch; ++j) {
+                const int k8 = lane + 32 * (j0 + j);
+                wb[j] = k8 < n8 ? __ldg(w + k8) : make_uint4(0, 0, 0, 0);
+            }
         }
 #pragma unroll
-        for (int e = 0; e < kGemvEpisodes; ++e) {
-            if (e >= E) break;
-            const float4 x0 = ld_dep(c4 + (size_t)e * (d / 4) + 2 * k8), x1 = ld_dep(c4 + (size_t)e * (d / 4) + 2 * k8 + 1);
-            float a = acc[e];
-            a = fmaf(wf[0], x0.x, a);
-            a = fmaf(wf[1], x0.y, a);
-            a = fmaf(wf[2], x0.z, a);
-            a = fmaf(wf[3], x0.w, a);
-            a = fmaf(wf[4], x1.x, a);
-            a = fmaf(wf[5], x1.y, a);
-            a = fmaf(wf[6], x1.z, a);
-            a = fmaf(wf[7], x1.w, a);
-            acc[e] = a;
+        for (int j = 0; j < kGemvBatch; ++j) {
+            const int k8 = lane + 32 * (j0 + j);
+            if (k8 >= n8) break;
+            const __nv_bfloat162 *wp = reinterpret_cast<const __nv_bfloat162 *>(&wb[j]);
+            float wf[8];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const float2 t = __bfloat1622float2(wp[i]);
+                wf[2 * i] = t.x;
+                wf[2 * i + 1] = t.y;
+            }
+#pragma unroll
+            for (int e = 0; e < kGemvEpisodes; ++e) {
+                if (e >= E) break;
+                const float4 x0 = csm[e * (d / 4) + 2 * k8], x1 = csm[e * (d / 4) + 2 * k8 + 1];
+                float a = acc[e];
+                a = fmaf(wf[0], x0.x, a);
+                a = fmaf(wf[1], x0.y, a);
+                a = fmaf(wf[2], x0.z, a);
+                a = fmaf(wf[3], x0.w, a);
+                a = fmaf(wf[4], x1.x, a);
+                a = fmaf(wf[5], x1.y, a);
+                a = fmaf(wf[6], x1.z, a);
+                a = fmaf(wf[7], x1.w, a);
+                acc[e] = a;
+            }
         }
     }
 #pragma unroll
@@ -593,10 +632,15 @@ static cudaError_t launch_router_t(const CompressArgs &a)
             *W2 = (const T *)a.W2;
     cudaError_t err = launch_lang_pool(a);
     if (err != cudaSuccess) return err;
-    if (sizeof(T) == 2 && E <= kGemvEpisodes && d % 8 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
-        err = launch_pdl(k_lang_bias_gemv, dim3((F + 7) / 8, L), dim3(256), 0, a.stream,
-                         (const __nv_bfloat16 *)a.W1, a.b1, (const float *)a.ws.lang_ctx, E, d, C, F, a.alpha_lang,
-                         a.ws.lang_bias);
+    const size_t gemv_smem = (size_t)E * d * sizeof(float);
+    if (sizeof(T) == 2 && E <= kGemvEpisodes && d % 8 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0 &&
+        gemv_smem <= 200 * 1024) {
+        err = cudaFuncSetAttribute(k_lang_bias_gemv, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)gemv_smem);
+        if (err == cudaSuccess)
+            err = launch_pdl(k_lang_bias_gemv, dim3((F + 7) / 8, L), dim3(256), gemv_smem, a.stream,
+                             (const __nv_bfloat16 *)a.W1, a.b1, (const float *)a.ws.lang_ctx, E, d, C, F,
+                             a.alpha_lang, a.ws.lang_bias);
+    }
     else if (sizeof(T) == 2 && d % 512 == 0 && C % 8 == 0 && ((uintptr_t)a.W1 & 15) == 0)
         err = launch_pdl(k_lang_bias_mma<8>, dim3((F + 63) / 64 * 8, (E + 63) / 64, L), dim3(128), 0, a.stream,
                          (const __nv_bfloat16 *)a.W1, a.b1, (const float *)a.ws.lang_ctx, E, d, C, F, a.alpha_lang,
