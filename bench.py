@@ -641,29 +641,36 @@ def run_ours(args):
     lat_graph = time_latency(graph1.replay)
     del graph1
 
-    # ---- one robot-control step: a single episode through all 32 layers
-    # (128 visual tokens keeping 4 of 16 groups, 48 language tokens), eager
-    # calls, L2 flushed before each step ------------------------------------
-    wl2 = synth.c2(128, 4)
-    inp2 = synth.gen_inputs(wl2)
-    rs2 = rolesub.RoleSub(wl2.L, wl2.H, wl2.dh, wl2.G, wl2.C, wl2.F, wl2.dtype, wl2.n_tok_array(),
-                          wl2.k_array(), wl2.n_query_array(), device=dev)
-    d2 = {k: to_dev(v) for k, v in inp2.items()}
-    p2, i2 = rs2.new_outputs()
-    o2 = torch.empty((wl2.L, wl2.q_rows, wl2.d), dtype=rs2.tdtype, device=dev)
+    # ---- one robot-control step: a single episode through all 32 layers,
+    # eager calls, L2 flushed before each step: c2's point of 128 visual
+    # tokens keeping 4 of 16 groups + 48 language tokens, and c3's
+    # aggressive joint compression (64 visual at 2 of 16, 48 language at 4
+    # of 16, router near-ties) -----------------------------------------------
+    def single_episode_ms(wl_s):
+        inp_s = synth.gen_inputs(wl_s)
+        rs_s = rolesub.RoleSub(wl_s.L, wl_s.H, wl_s.dh, wl_s.G, wl_s.C, wl_s.F, wl_s.dtype, wl_s.n_tok_array(),
+                               wl_s.k_array(), wl_s.n_query_array(), device=dev)
+        d_s = {k: to_dev(v) for k, v in inp_s.items()}
+        p_s, i_s = rs_s.new_outputs()
+        o_s = torch.empty((wl_s.L, wl_s.q_rows, wl_s.d), dtype=rs_s.tdtype, device=dev)
 
-    def step2():
-        rs2.compress(d2["h"], d2["v"], d2["R"], d2["W_re"], d2["b_re"], d2["W1"], d2["b1"], d2["W2"], d2["b2"],
-                     wl2.alpha_role, wl2.alpha_lang, packed=p2, idx=i2)
-        rs2.attend(d2["q"], d2["K"], p2, i2, d2["R"], o=o2)
+        def step_s():
+            rs_s.compress(d_s["h"], d_s["v"], d_s["R"], d_s["W_re"], d_s["b_re"], d_s["W1"], d_s["b1"], d_s["W2"],
+                          d_s["b2"], wl_s.alpha_role, wl_s.alpha_lang, packed=p_s, idx=i_s)
+            rs_s.attend(d_s["q"], d_s["K"], p_s, i_s, d_s["R"], o=o_s)
 
-    for _ in range(3):
-        step2()
-    torch.cuda.synchronize()
-    ctl_ms = time_latency(step2)
-    code, _ = rs2.device_status()
-    assert code == 0, f"device status {code}"
-    del lat_flush, d2, rs2, p2, i2, o2
+        for _ in range(3):
+            step_s()
+        torch.cuda.synchronize()
+        ms = time_latency(step_s)
+        code, _ = rs_s.device_status()
+        assert code == 0, f"device status {code}"
+        return ms
+
+    wl2, wl3 = synth.c2(128, 4), synth.c3()
+    ctl_ms = single_episode_ms(wl2)
+    c3_ms = single_episode_ms(wl3)
+    del lat_flush
 
     # ---- end to end through the public API from pinned host buffers. The
     # layers go in chunks of E2E_CHUNK: a chunk's activations are copied in
@@ -781,6 +788,9 @@ def run_ours(args):
     control = {"workload": wl2.name, "describe": wl2.describe, "layers": wl2.L,
                "l2": "flushed before each step", "ms_per_step": ctl_ms,
                "query_tokens_per_s_per_layer": wl2.q_rows * wl2.L / (ctl_ms / 1e3)}
+    step_c3 = {"workload": wl3.name, "describe": wl3.describe, "layers": wl3.L,
+               "l2": "flushed before each step", "ms_per_step": c3_ms,
+               "query_tokens_per_s_per_layer": wl3.q_rows * wl3.L / (c3_ms / 1e3)}
     select = {"episodes": 64, "views": 2, "tokens_per_view": 256, "kept_per_view": sel_k, "ms": sel_ms,
               "l2": "flushed before each call",
               "algorithmic_bytes": sel_bytes, "GB/s": sel_bytes / (sel_ms / 1e3) / 1e9}
@@ -801,7 +811,7 @@ def run_ours(args):
                     "o_equals_whole_workload_call": e2e_same},
             "gpu_launches": launches,
             "roofline": roof, "compress": comp, "compress_additive": comp_add, "budget": budget,
-            "select_tokens": select, "latency_one_layer": latency, "control_step_c2": control, "dense_rotation": dense,
+            "select_tokens": select, "latency_one_layer": latency, "control_step_c2": control, "step_c3": step_c3, "dense_rotation": dense,
             "clocks": {"sm_mhz": clocks["sm_mhz"], "sm_max_mhz": clocks["sm_max_mhz"],
                        "reasons": clocks["reasons"], "samples": clocks["samples"]}}
     if ws == 1 and rank == 0 and not args.no_cpu_baseline:
